@@ -1,0 +1,152 @@
+"""Weight-only and KV-cache quantisers of the oracle (test infrastructure only).
+
+The paper lists INT8 and INT4 weight-only quantisation and an INT8 KV cache
+among its deployment configurations (Sec. 2 "LLM deployment configuration
+parameters"; Sec. 3.2; Table "Models and configurations") and states their
+memory effect (-50 % / -75 %, Sec. 3.2), but not their arithmetic.  The
+readings implemented here:
+
+int8 weights, per output channel (row n of W[N, K]):
+    a   = max_k |W[n, k]|                      (exact: bf16 inputs)
+    s_n = bf16 round-toward-+inf of fp32(a / 127)
+    q   = clamp(rint(fp32(W / s_n)), -127, 127)   rint = ties to even
+    dequantised weight = q * s_n;  a zero row gives s = 0, q = 0.
+
+int4 weights, asymmetric, groups of 128 along K (row n, group g):
+    mn = min(0, min w), mx = max(0, max w)
+    s  = bf16 round-toward-+inf of fp32(fp32(mx - mn) / 15)
+    z  = clamp(rint(fp32(-mn / s)), 0, 15)     (stored as bf16, exact)
+    q  = clamp(rint(fp32(w / s)) + z, 0, 15)
+    dequantised weight = (q - z) * s;  a zero range gives s = z = q = 0.
+    Packing: bytes [N][K/2]; element 2j in the low nibble, 2j+1 in the high.
+
+int8 KV cache, per token and per KV head, separately for K (after RoPE) and V:
+    s = fp32(max |x| / 127) (stored as fp32), q = clamp(rint(fp32(x / s)), -127, 127)
+    dequantised value = q * s;  s = 0 gives q = 0.
+
+Every division and rounding decision is taken in IEEE fp32, as the device
+does, so codes, packing and scales can be compared bit for bit.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+GROUP = 128
+
+
+def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit patterns (uint16) to their exact fp32 values."""
+    return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def f32_to_bf16_rne(x: np.ndarray) -> np.ndarray:
+    """fp32 -> bf16 bits, round to nearest, ties to even (finite inputs)."""
+    b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    b = b + np.uint64(0x7FFF) + ((b >> np.uint64(16)) & np.uint64(1))
+    return (b >> np.uint64(16)).astype(np.uint16)
+
+
+def f32_to_bf16_ceil(x: np.ndarray) -> np.ndarray:
+    """Non-negative fp32 -> bf16 bits, rounded toward +inf (smallest bf16 >= x)."""
+    b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    up = (b & np.uint64(0xFFFF)) != 0
+    hi = b >> np.uint64(16)
+    return (hi + up.astype(np.uint64)).astype(np.uint16)
+
+
+# ---------------------------------------------------------------- int8 weights
+def quantize_int8_rows(w_bits: np.ndarray):
+    """int8 per-output-channel absmax quantiser.
+
+    w_bits: bf16 bit patterns [N, K].  Returns (codes int8 [N, K],
+    scale bf16 bits uint16 [N]).
+    """
+    w = bf16_to_f32(w_bits)
+    amax = np.max(np.abs(w), axis=1)
+    s = bf16_to_f32(f32_to_bf16_ceil(amax / np.float32(127.0)))
+    with np.errstate(divide="ignore", invalid="ignore"):
+        r = np.where(s[:, None] > 0, w / s[:, None], np.float32(0.0)).astype(np.float32)
+    q = np.clip(np.rint(r), -127, 127).astype(np.int8)
+    return q, f32_to_bf16_ceil(s)  # s is already a bf16 value: ceil is the identity
+
+
+def dequant_int8(codes: np.ndarray, scale_bits: np.ndarray) -> np.ndarray:
+    return codes.astype(np.float64) * bf16_to_f32(scale_bits).astype(np.float64)[:, None]
+
+
+# ---------------------------------------------------------------- int4 weights
+def quantize_int4_g128(w_bits: np.ndarray):
+    """int4 asymmetric group-128 quantiser.
+
+    w_bits: bf16 bit patterns [N, K], K % 128 == 0.  Returns (packed uint8
+    [N, K/2], scale bf16 bits [N, K/128], zero bf16 bits [N, K/128]).
+    """
+    n, k = w_bits.shape
+    assert k % GROUP == 0
+    w = bf16_to_f32(w_bits).reshape(n, k // GROUP, GROUP)
+    mn = np.minimum(np.float32(0.0), w.min(axis=2))
+    mx = np.maximum(np.float32(0.0), w.max(axis=2))
+    d = (mx - mn).astype(np.float32)
+    s = bf16_to_f32(f32_to_bf16_ceil((d / np.float32(15.0)).astype(np.float32)))
+    pos = s > 0
+    with np.errstate(divide="ignore", invalid="ignore"):
+        zr = np.where(pos, (-mn) / s, np.float32(0.0)).astype(np.float32)
+        r = np.where(pos[..., None], w / s[..., None], np.float32(0.0)).astype(np.float32)
+    z = np.clip(np.rint(zr), 0, 15)
+    q = np.clip(np.rint(r) + z[..., None], 0, 15).astype(np.uint8).reshape(n, k)
+    packed = (q[:, 0::2] | (q[:, 1::2] << np.uint8(4))).astype(np.uint8)
+    return packed, f32_to_bf16_rne(s), f32_to_bf16_rne(z.astype(np.float32))
+
+
+def unpack_int4(packed: np.ndarray) -> np.ndarray:
+    """[N, K/2] bytes -> [N, K] codes 0..15 (low nibble = even element)."""
+    n, kh = packed.shape
+    q = np.empty((n, kh * 2), dtype=np.uint8)
+    q[:, 0::2] = packed & np.uint8(0x0F)
+    q[:, 1::2] = packed >> np.uint8(4)
+    return q
+
+
+def dequant_int4(packed, scale_bits, zero_bits) -> np.ndarray:
+    q = unpack_int4(packed).astype(np.float64)
+    n, k = q.shape
+    s = bf16_to_f32(scale_bits).astype(np.float64)
+    z = bf16_to_f32(zero_bits).astype(np.float64)
+    q = q.reshape(n, k // GROUP, GROUP)
+    return ((q - z[..., None]) * s[..., None]).reshape(n, k)
+
+
+# ---------------------------------------------------------------- int8 KV cache
+def quantize_kv_int8(x_bits: np.ndarray):
+    """Per-row (token, KV head) absmax int8 quantiser over the last axis.
+
+    x_bits: bf16 bit patterns [..., hd].  Returns (codes int8 [..., hd],
+    scale fp32 [...]).
+    """
+    x = bf16_to_f32(x_bits)
+    s = (np.max(np.abs(x), axis=-1) / np.float32(127.0)).astype(np.float32)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        r = np.where(s[..., None] > 0, x / s[..., None], np.float32(0.0)).astype(np.float32)
+    q = np.clip(np.rint(r), -127, 127).astype(np.int8)
+    return q, s
+
+
+def dequant_kv_int8(codes: np.ndarray, scales: np.ndarray) -> np.ndarray:
+    return codes.astype(np.float64) * scales.astype(np.float64)[..., None]
+
+
+# ---------------------------------------------------------------- one entry point
+def quantize_weight(w_bits: np.ndarray, wquant: int):
+    """wquant 0 = bf16 (no codes), 1 = int8 per channel, 2 = int4 group 128.
+
+    Returns (payload dict, dequantised fp64 matrix).
+    """
+    if wquant == 0:
+        return {"w": w_bits}, bf16_to_f32(w_bits).astype(np.float64)
+    if wquant == 1:
+        q, s = quantize_int8_rows(w_bits)
+        return {"codes": q, "scales": s}, dequant_int8(q, s)
+    if wquant == 2:
+        p, s, z = quantize_int4_g128(w_bits)
+        return {"codes": p, "scales": s, "zeros": z}, dequant_int4(p, s, z)
+    raise ValueError(wquant)
