@@ -92,7 +92,8 @@ def quantize_int4_g128(w_bits: np.ndarray):
     with np.errstate(divide="ignore", invalid="ignore"):
         zr = np.where(pos, (-mn) / s, np.float32(0.0)).astype(np.float32)
         r = np.where(pos[..., None], w / s[..., None], np.float32(0.0)).astype(np.float32)
-    z = np.clip(np.rint(zr), 0, 15)
+    # the zero point is an integer in [0, 15]; "+ 0" turns rint(-0.0) into +0
+    z = np.clip(np.rint(zr), 0, 15) + np.float32(0.0)
     q = np.clip(np.rint(r) + z[..., None], 0, 15).astype(np.uint8).reshape(n, k)
     packed = (q[:, 0::2] | (q[:, 1::2] << np.uint8(4))).astype(np.uint8)
     return packed, f32_to_bf16_rne(s), f32_to_bf16_rne(z.astype(np.float32))

@@ -118,8 +118,9 @@ def test_int4_codes_nearest_and_bounded():
             best = np.abs(seg[:, None] - (cand[None, :] - zg) * sg).min(axis=1)
             assert np.all(mine <= best + 2.0 ** -22 * max(sg, 1e-30) * 16)
             assert np.all(mine <= sg / 2 * (1 + 2.0 ** -20))
-    # zero row -> s = z = q = 0
+    # zero row -> s = z = q = 0; the stored zero point is +0 (an integer, no sign)
     assert np.all(s[0] == 0) and np.all(z[0] == 0) and np.all(q[0] == 0)
+    assert np.all(z_bits >> 15 == 0)
 
 
 def test_int4_packing_order_and_roundtrip():
