@@ -1,0 +1,346 @@
+"""Benchmark of the fingerprint forward pass on GB300 (one JSON line on rank 0).
+
+A step is one request batch through the whole hot path: prefill of the
+batch's prompts, then greedy decode steps (the decode step is a replayed CUDA
+graph).  The default workload is the Llama-2-7B-shaped fingerprint:
+2 decoder blocks (d 4096, 32 heads x 128, FFN 11008, vocab 32000), int8
+per-channel weight-only quantisation, bf16 KV cache, batch 8, 512-token
+prompts, 100 generated tokens.  Weights are synthetic (SplitMix64 /
+Irwin-Hall N(0, 0.02), drawn on the device), prompts are seeded uniform ids.
+
+value      decode tokens/s over all ranks = ranks * batch * decode steps / max-over-ranks
+           device time of the decode phases (CUDA events on the library's stream)
+e2e        the same metric through the C ABI with host buffers: prompt H2D from
+           pinned memory each step and the token D2H after every decode step
+roofline   the dominant decode kernel: algorithmic bytes per launch / mean launch
+           duration (CUDA events between kernels, instrumented decode steps)
+cpu_baseline  the oracle (numpy, fp64) on the host cores, a bounded sample
+
+--impl reference times the oracle alone as the reference arm.
+Multi-GPU: one independent replica per rank (the path does not shard).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decode tokens/s and achieved HBM GB/s per fingerprint block; prefill TFLOP/s"
+
+# name: (n_layers, hidden, heads, kv heads, head_dim, ffn, vocab), wquant, kvquant, batch, prompt, decode
+CONFIGS = {
+    "tiny": ((1, 512, 8, 8, 64, 1376, 32000), 0, 0, 1, 32, 16),
+    "l7b": ((2, 4096, 32, 32, 128, 11008, 32000), 1, 0, 8, 512, 100),
+    "l13b": ((2, 5120, 40, 40, 128, 13824, 32000), 2, 0, 16, 1024, 100),
+    "l70b": ((2, 8192, 64, 8, 128, 28672, 32000), 2, 1, 32, 2048, 100),
+}
+WQ_NAME = {0: "bf16", 1: "int8-per-channel", 2: "int4-g128"}
+KV_NAME = {0: "bf16", 1: "int8-per-token-head"}
+
+
+def arch_dict(t):
+    keys = ("n_layers", "hidden", "n_heads", "n_kv_heads", "head_dim", "ffn", "vocab")
+    d = dict(zip(keys, t))
+    d.update(rms_eps=1e-5, rope_base=10000.0)
+    return d
+
+
+# ---------------------------------------------------------------- byte model
+def mat_bytes(n, k, wq):
+    return {0: 2 * n * k, 1: n * k + 2 * n, 2: n * k // 2 + 4 * n * (k // 128)}[wq]
+
+
+def kernel_bytes(a, wq, kvq, B, ctx):
+    """Algorithmic HBM bytes of one launch of each decode kernel class:
+    weight codes + scales/zeros + activations in and out (+ K/V rows read)."""
+    d, f, V = a["hidden"], a["ffn"], a["vocab"]
+    qd = a["n_heads"] * a["head_dim"]
+    kvd = a["n_kv_heads"] * a["head_dim"]
+    nqkv = qd + 2 * kvd
+    kv_tok = 2 * kvd * 2 if kvq == 0 else 2 * kvd + 2 * a["n_kv_heads"] * 4
+    return {
+        "lin_qkv": mat_bytes(nqkv, d, wq) + 2 * B * (d + nqkv),
+        "lin_o": mat_bytes(d, qd, wq) + 2 * B * (qd + 2 * d),
+        "lin_gu": mat_bytes(2 * f, d, wq) + 2 * B * (d + f),
+        "lin_down": mat_bytes(d, f, wq) + 2 * B * (f + 2 * d),
+        "lm_head": 2 * V * d + 2 * B * d + 4 * B * V,
+        "attn": B * ctx * kv_tok + 2 * B * 2 * qd,
+    }
+
+
+# ---------------------------------------------------------------- clocks
+CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+           "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+           "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={CLOCK_Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+        return False
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- oracle timing
+def oracle_sample(cfg, batch, steps, decode_tokens):
+    """Time the oracle (numpy fp64, test infrastructure) on the same workload:
+    the full config shape at the same batch and prompt; the prompt's prefill
+    is set-up, each timed step is ``decode_tokens`` greedy decode steps.
+    Returns (tokens/s, seconds per step list, description)."""
+    import synth
+    from oracle import model as M
+
+    t, wq, kvq, B, S, N = cfg
+    arch = M.Arch(*t)
+    get = lambda l, k, shape: (synth.f32_to_bf16_bits(np.ones(shape, np.float32)) if len(shape) == 1
+                               else synth.weight_bf16(0, l, k, shape))
+    w, _ = M.build_weights(arch, wq, get)
+    ref = M.Fingerprint(arch, w, kvq, batch, S + steps * decode_tokens + 1)
+    toks = synth.tokens(0, batch * S, arch.vocab).reshape(batch, S)
+    out = ref.prefill(toks)
+    tok = out["tokens"]
+    times = []
+    for _ in range(steps):
+        t0 = time.perf_counter()
+        for _ in range(decode_tokens):
+            tok = ref.decode(tok)["tokens"]
+        times.append(time.perf_counter() - t0)
+    tps = batch * decode_tokens * steps / sum(times)
+    desc = (f"oracle decode, batch {batch}, prompt {S} (prefill untimed), {decode_tokens} tokens x {steps} "
+            f"timed steps, fp64 numpy")
+    return tps, times, desc
+
+
+def blas_threads():
+    try:
+        from threadpoolctl import threadpool_info
+
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def run_reference(args, cfg):
+    """Reference arm: the oracle on the host cores (rank 0 only)."""
+    if int(os.environ.get("RANK", "0")) != 0:
+        return 0
+    t, wq, kvq, B, S, N = cfg
+    tps, times, desc = oracle_sample(cfg, B, args.warmup + args.steps, 2)
+    times = times[args.warmup:]
+    tps = B * 2 * len(times) / sum(times)
+    line = {
+        "metric": METRIC, "value": tps, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+        "config": config_json(args, cfg),
+        "cpu_baseline": {"value": tps, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": tps, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_json(args, cfg):
+    t, wq, kvq, B, S, N = cfg
+    a = arch_dict(t)
+    return {"workload": f"{args.config}-shaped fingerprint", "layers": a["n_layers"], "hidden": a["hidden"],
+            "heads": a["n_heads"], "kv_heads": a["n_kv_heads"], "head_dim": a["head_dim"], "ffn": a["ffn"],
+            "vocab": a["vocab"], "weights": WQ_NAME[wq], "kv_cache": KV_NAME[kvq], "batch": B, "prompt": S,
+            "decode_tokens": N, "parallelism": f"replicas{args.gpus}",
+            "l2": "inputs larger than L2 (every decode step streams all block weights and the LM head)"}
+
+
+# ---------------------------------------------------------------- our arm
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="l7b", choices=list(CONFIGS))
+    ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass (profiling runs)")
+    args = ap.parse_args()
+    cfg = CONFIGS[args.config]
+    if args.impl == "reference":
+        return run_reference(args, cfg)
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_2501_13111_gb300 as fp
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    t, wq, kvq, B, S, N = cfg
+    a = arch_dict(t)
+    stream = torch.cuda.Stream()
+    h = fp.fp_create(a, wq, kvq, B, S + N + 1, seed=0, stream=stream.cuda_stream)
+    try:
+        fp.fp_load_prompt(h, None, S)
+        for _ in range(args.warmup):
+            fp.fp_prefill(h, None, want_next=False, prompt_len=S)
+            fp.fp_decode_steps(h, N)
+        torch.cuda.synchronize()
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+        barrier()
+        torch.cuda.synchronize()
+        with ClockSampler(local) as clk:
+            for k in range(args.steps):
+                ev[k][0].record(stream)
+                fp.fp_prefill(h, None, want_next=False, prompt_len=S)
+                ev[k][1].record(stream)
+                fp.fp_decode_steps(h, N)
+                ev[k][2].record(stream)
+            torch.cuda.synchronize()
+        barrier()
+        ttft = [ev[k][0].elapsed_time(ev[k][1]) for k in range(args.steps)]
+        dec = [ev[k][1].elapsed_time(ev[k][2]) for k in range(args.steps)]
+        total_ms = max_over_ranks(sum(ttft) + sum(dec))
+        dec_ms = max_over_ranks(sum(dec))
+        ttft_ms = max_over_ranks(sum(ttft) / args.steps)
+        value = world * B * N * args.steps / (dec_ms * 1e-3)
+
+        # instrumented decode steps: per-block and per-kernel device time
+        prof = fp.fp_profile(h, S, N, warmup=0, iters=1).as_dict()
+        mean_ctx = S + (min(N, 8) + 1) / 2.0
+        kb = kernel_bytes(a, wq, kvq, B, mean_ctx)
+        cls_time = {c: prof["kernel_ms"][c] for c in kb}
+        dom = max(cls_time, key=cls_time.get)
+        per_launch_ms = cls_time[dom] / max(1, prof["kernel_launches"][dom])
+        achieved = kb[dom] / (per_launch_ms * 1e-3) / 1e9
+        peaks = {}
+        pk = os.path.join(ROOT, "MEASURED_PEAKS.json")
+        if os.path.exists(pk):
+            peaks = json.load(open(pk))
+        peak, peak_src = (peaks["hbm_gbs"], "measured") if "hbm_gbs" in peaks else (6800.0, "fallback")
+        block_gbs = [bb / (bm * 1e-3) / 1e9 for bb, bm in zip(prof["block_bytes"], prof["block_ms"])]
+        launches = args.steps * (prof["prefill_launches"] + N * prof["decode_launches"])
+
+        # end to end through the C ABI with host buffers
+        e2e = None
+        if not args.no_e2e:
+            pin_prompt = torch.empty((B, S), dtype=torch.int32, pin_memory=True)
+            host_prompt = pin_prompt.numpy()
+            import synth
+
+            host_prompt[:] = synth.tokens(0, B * S, a["vocab"]).reshape(B, S)
+            pin_out = torch.empty(B, dtype=torch.int32, pin_memory=True).numpy()
+            fp.fp_prefill(h, host_prompt, out=pin_out)
+            for _ in range(N):
+                fp.fp_decode_step(h, None, out=pin_out)
+            barrier()
+            t_dec = 0.0
+            for _ in range(args.steps):
+                fp.fp_prefill(h, host_prompt, out=pin_out)
+                t0 = time.perf_counter()
+                for _ in range(N):
+                    fp.fp_decode_step(h, None, out=pin_out)
+                t_dec += time.perf_counter() - t0
+            barrier()
+            t_dec = max_over_ranks(t_dec)
+            e2e = {"value": world * B * N * args.steps / t_dec, "unit": "tokens/s",
+                   "h2d_bytes_per_step": B * S * 4, "d2h_bytes_per_step": B * 4 * (N + 1)}
+
+        cpu = None
+        if rank == 0 and world == 1 and not args.no_cpu_baseline:
+            tps, times, desc = oracle_sample(cfg, B, 2, 2)
+            cpu = {"value": tps, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle", "sample": desc}
+
+        if rank == 0:
+            line = {
+                "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+                "data": "synthetic (seeded weights and prompts)", "config": config_json(args, cfg),
+                "ttft_ms": ttft_ms, "tpot_ms": dec_ms / (args.steps * N),
+                "prefill_tflops": prof["prefill_flops"] / (ttft_ms * 1e-3) / 1e12,
+                "block_hbm_gbs": block_gbs, "block_ms": prof["block_ms"],
+                "peak_hbm_bytes": prof["peak_hbm_bytes"], "weight_bytes": prof["weight_bytes"],
+                "kernel_ms_per_step": prof["kernel_ms"],
+                "roofline": {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peak,
+                             "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
+                             "bytes_per_launch": kb[dom], "launch_ms": per_launch_ms, "traffic": None},
+                "gpu_launches": launches,
+                "clocks": clk.summary(),
+                "e2e": e2e,
+                "cpu_baseline": cpu,
+            }
+            print(json.dumps(line), flush=True)
+    finally:
+        fp.fp_destroy(h)
+        if world > 1:
+            dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

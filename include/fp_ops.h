@@ -1,0 +1,131 @@
+/*
+ * fp_ops.h -- one C entry point per step of the fingerprint forward pass.
+ *
+ * These are the kernels the fingerprint runtime (fp.h) strings together,
+ * exposed one by one on caller-owned DEVICE buffers so each step can be
+ * checked against the oracle and timed alone.  Steps follow the decoder
+ * block the fingerprint keeps from its LLM (arXiv 2501.13111, Sec. 1 "Our
+ * work", Sec. 5.1) under the deployment configurations of Sec. 3.2 (weight
+ * and KV-cache quantisation).
+ *
+ * Conventions:
+ *   - Every pointer argument is a device pointer unless its name starts
+ *     with host_.  Buffers are row-major; bf16 is passed as its uint16 bits.
+ *   - The launch is asynchronous on `stream` (cudaStream_t, NULL = legacy
+ *     default stream).  Arguments are checked on the host before any launch:
+ *     FP_ERR_INVALID_ARG / FP_ERR_UNSUPPORTED and nothing is launched.
+ *     FP_ERR_CUDA if the launch itself fails.  Nothing is allocated.
+ *   - Output buffers must not overlap inputs unless a function says so.
+ *   - Return codes are the FP_* codes of fp.h.
+ */
+#ifndef FP_OPS_H
+#define FP_OPS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include "fp.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Quantise a bf16 weight matrix w [N][K] into the wquant format of fp.h
+ * (Sec. 3.2; formats in fp.h).  int8: codes int8 [N][K], scales bf16 [N].
+ * int4: codes uint8 [N][K/2], scales and zeros bf16 [N][K/128]; K % 128 == 0.
+ * bf16: codes receives a copy of w.  Codes are bit-exact with the reading
+ * (fp32 IEEE division, round half to even). */
+int fp_op_quantize(int wquant, const uint16_t* w, int N, int K, void* codes, uint16_t* scales,
+                   uint16_t* zeros, void* stream);
+
+/* Fill w [n] with the seeded bf16 weights of stream `stream_id` (SplitMix64
+ * counter-based draws, Irwin-Hall(4), sigma 0.02; elements start..start+n-1). */
+int fp_op_init_weights(uint16_t* w, long long n, unsigned long long seed, long long stream_id,
+                       long long start, void* stream);
+
+/* Epilogues of fp_op_linear. */
+enum {
+  FP_EPI_STORE = 0,  /* y bf16 [M][N]                                          */
+  FP_EPI_RESID = 1,  /* y bf16 [M][N] = residual + x W^T; residual may equal y  */
+  FP_EPI_SWIGLU = 2, /* W rows = [gate (N/2 rows); up (N/2 rows)];
+                        y bf16 [M][N/2] = silu(x Wg^T) * (x Wu^T)             */
+  FP_EPI_F32 = 3     /* y fp32 [M][N]                                          */
+};
+
+/* Weight-only linear y = x W^T (the "linear layers" of the block) with the
+ * dequantisation fused: x bf16 [M][K]; W in the wquant format of fp.h
+ * (codes / scales / zeros as fp_op_quantize writes them); fp32 accumulation.
+ * Kernel choice depends on M only (decode GEMV for small M, tensor-core GEMM
+ * otherwise).  workspace: see fp_op_linear_workspace_bytes (may be NULL if
+ * that returns 0). */
+int fp_op_linear(int wquant, int epilogue, const uint16_t* x, int M, int N, int K, const void* codes,
+                 const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                 void* workspace, size_t workspace_bytes, void* stream);
+size_t fp_op_linear_workspace_bytes(int wquant, int M, int N, int K);
+
+/* RMSNorm of selected rows: y[r] = x[r*row_stride + row_offset] /
+ * sqrt(mean(x^2) + eps) * g, r < M; x, y, g bf16; fp32 arithmetic. */
+int fp_op_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int row_offset, const uint16_t* g,
+                  float eps, uint16_t* y, void* stream);
+
+/* Embedding gather h[m] = E[tok[m]]; tok int32 [M], E bf16 [V][d].  An id
+ * outside [0, V) writes a zero row and sets *err = 1 (err may be NULL). */
+int fp_op_embed(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h, int32_t* err,
+                void* stream);
+
+/* Paged KV cache view.  Pools are [n_pages][n_kv_heads][page_size][head_dim]
+ * (bf16 or int8 codes); scales (int8 only) fp32 [n_pages][n_kv_heads][page_size];
+ * page_table int32 [batch][pages_per_seq]: position p of sequence b lives in
+ * page page_table[b][p / page_size], slot p % page_size. */
+typedef struct fp_kv_view {
+  int kvquant, n_kv_heads, head_dim, page_size, pages_per_seq, n_pages;
+  void* k_pool;
+  void* v_pool;
+  float* k_scale;
+  float* v_scale;
+  const int32_t* page_table;
+} fp_kv_view;
+
+/* RoPE table for positions 0..max_pos-1: cs fp32 [max_pos][head_dim/2][2] =
+ * (cos, sin) of p * base^(-2i/hd), computed on the host in fp64 and rounded
+ * to fp32, then copied to the device (synchronous). */
+int fp_op_rope_table(int max_pos, int head_dim, float base, float* cs, void* stream);
+
+/* RoPE + KV-cache append.  qkv bf16 [B*S][row_stride]: per token, H query
+ * heads, then Hkv key heads, then Hkv value heads, head_dim each.  Token s
+ * of sequence b sits at position pos[b] + s.  Query and key heads are
+ * rotated (rotate-half); queries are written back in place; keys (rotated,
+ * rounded to bf16) and values go to the cache, quantised per (token, KV
+ * head) when kvquant is int8.  rope_cs (fp_op_rope_table) must cover
+ * pages_per_seq * page_size positions.  A position outside
+ * [0, pages_per_seq * page_size) or a page id outside the pool sets
+ * *err = 1 (err may be NULL) and skips that head. */
+int fp_op_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_heads, const fp_kv_view* kv,
+                  const int32_t* pos, const float* rope_cs, int32_t* err, void* stream);
+
+/* Decode attention: one query row per sequence, q bf16 [B][q_stride] (head h
+ * at h*head_dim), attends over positions 0 .. len[b]-1 of the cache
+ * (softmax(q K^T / sqrt(hd)) V, query head j reads KV head j / (H/Hkv));
+ * out bf16 [B][n_heads*head_dim].  Split over the context in chunks; the
+ * partial results go to `workspace` (fp_op_attention_decode_workspace_bytes
+ * for at most max_len cached positions) and a second kernel combines them.
+ * len[b] in [1, max_len]; a larger len[b] is clipped to max_len and sets
+ * *err = 1 (err may be NULL). */
+int fp_op_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, const fp_kv_view* kv,
+                           const int32_t* len, int max_len, uint16_t* out, void* workspace,
+                           size_t workspace_bytes, int32_t* err, void* stream);
+size_t fp_op_attention_decode_workspace_bytes(int B, int n_heads, int head_dim, int max_len);
+
+/* Prefill attention: causal, S query rows per sequence at positions 0..S-1,
+ * q bf16 [B*S][q_stride]; keys/values read from the cache positions 0..S-1;
+ * out bf16 [B*S][n_heads*head_dim]. */
+int fp_op_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
+                            const fp_kv_view* kv, uint16_t* out, int32_t* err, void* stream);
+
+/* Greedy choice out[m] = argmax logits[m][:V] (fp32); ties to the lowest id. */
+int fp_op_argmax(const float* logits, int M, int V, int32_t* out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FP_OPS_H */

@@ -1,0 +1,230 @@
+// Row-wise kernels of the fingerprint block: embedding gather, RMSNorm,
+// RoPE + KV-cache append (with the int8 KV quantiser fused into the cache
+// write), greedy argmax and the position counter.
+//
+// Components: embedding, normalisation and the LM head's greedy choice are
+// among the fingerprint's components (Sec. 1 "Our work"; Sec. 5.1); the KV
+// cache and its INT8 variant are a deployment configuration (Sec. 2, Sec. 3.2,
+// table "Models and configurations"); the KV cache keeps per-token decode
+// cost constant (Sec. 5.3, before Eq. 1).
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace fpk {
+
+// ------------------------------------------------------------------ embedding
+// One CTA per token row; 16-byte copies (d % 8 == 0).
+__global__ void embed_kernel(const int32_t* __restrict__ tok, const uint16_t* __restrict__ E, int V, int d,
+                             uint16_t* __restrict__ h, int32_t* err) {
+  const long long m = blockIdx.x;
+  int t = tok[m];
+  uint4* dst = reinterpret_cast<uint4*>(h + m * d);
+  const int chunks = d / 8;
+  if (t < 0 || t >= V) {
+    if (threadIdx.x == 0 && err) atomicExch(err, 1);
+    for (int c = threadIdx.x; c < chunks; c += blockDim.x) dst[c] = make_uint4(0, 0, 0, 0);
+    return;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(E + (long long)t * d);
+  for (int c = threadIdx.x; c < chunks; c += blockDim.x) dst[c] = ld_nc16(src + c);
+}
+
+cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h, int32_t* err,
+                         cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  embed_kernel<<<M, 128, 0, s>>>(tok, E, V, d, h, err);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ RMSNorm
+// y[r] = x[r * stride + offset] * rsqrt(mean(x^2) + eps) * g, fp32 math.
+// One CTA of 128 threads per row; 16-byte loads (d % 8 == 0).
+__global__ void rmsnorm_kernel(const uint16_t* __restrict__ x, int d, int row_stride, int row_offset,
+                               const uint16_t* __restrict__ g, float eps, uint16_t* __restrict__ y) {
+  const long long r = blockIdx.x;
+  const uint4* xr = reinterpret_cast<const uint4*>(x + ((long long)r * row_stride + row_offset) * d);
+  const uint4* gr = reinterpret_cast<const uint4*>(g);
+  uint4* yr = reinterpret_cast<uint4*>(y + r * d);
+  const int chunks = d / 8;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+    uint4 v = xr[c];
+    uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 f = bf2x2f(w[i]);
+      ss += f.x * f.x + f.y * f.y;
+    }
+  }
+  ss = warp_sum(ss);
+  __shared__ float red[4];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = red[0] + red[1] + red[2] + red[3];
+  float inv = rsqrtf(tot / (float)d + eps);
+  for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+    uint4 v = xr[c], gg = gr[c];
+    uint32_t w[4] = {v.x, v.y, v.z, v.w}, gw[4] = {gg.x, gg.y, gg.z, gg.w}, o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float2 f = bf2x2f(w[i]), gf = bf2x2f(gw[i]);
+      o[i] = pack_bf2(f.x * inv * gf.x, f.y * inv * gf.y);
+    }
+    yr[c] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+cudaError_t launch_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int row_offset, const uint16_t* g,
+                           float eps, uint16_t* y, cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  rmsnorm_kernel<<<M, 128, 0, s>>>(x, d, row_stride, row_offset, g, eps, y);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ argmax
+// One CTA per row; ties go to the lowest index.
+__global__ void argmax_kernel(const float* __restrict__ logits, int V, int32_t* __restrict__ out) {
+  const float* lr = logits + (long long)blockIdx.x * V;
+  float best = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int i = threadIdx.x; i < V; i += blockDim.x) {
+    float v = lr[i];
+    if (v > best) { best = v; bi = i; }  // i increases per thread: strict > keeps the first
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    float ov = __shfl_xor_sync(0xffffffffu, best, o);
+    int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
+  }
+  __shared__ float sv[32];
+  __shared__ int si[32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) { sv[warp] = best; si[warp] = bi; }
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    best = lane < nw ? sv[lane] : -INFINITY;
+    bi = lane < nw ? si[lane] : 0x7fffffff;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      float ov = __shfl_xor_sync(0xffffffffu, best, o);
+      int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
+    }
+    if (lane == 0) out[blockIdx.x] = bi == 0x7fffffff ? 0 : bi;
+  }
+}
+
+cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  argmax_kernel<<<M, 512, 0, s>>>(logits, V, out);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ RoPE + KV append
+// One warp per (token, head slot); slots are the H query heads, then the Hkv
+// key heads, then the Hkv value heads.  Lane l holds elements l + 32 j, so
+// each rotate-half pair (i, i + hd/2) sits in one lane.  Rotation in fp32,
+// rounded to bf16.  Keys and values go to the paged cache; with an int8
+// cache each (token, KV head) row is quantised: s = fp32(max|x| / 127),
+// q = clamp(rint(fp32(x / s)), -127, 127).
+template <int HD, int KVQ>
+__global__ void rope_kv_kernel(uint16_t* __restrict__ qkv, int B, int S, int row_stride, int H, fp_kv_view kv,
+                               const int32_t* __restrict__ pos, const float* __restrict__ cs, int32_t* err) {
+  constexpr int E = HD / 32;
+  const int Hkv = kv.n_kv_heads;
+  const int slots = H + 2 * Hkv;
+  const long long wid = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (wid >= (long long)B * S * slots) return;
+  const int lane = threadIdx.x & 31;
+  const int slot = (int)(wid % slots);
+  const long long m = wid / slots;
+  const int b = (int)(m / S), s = (int)(m % S);
+  const int p = pos[b] + s;
+  const int lp = p / kv.page_size;
+  if (p < 0 || lp >= kv.pages_per_seq) {  // outside the cache and the RoPE table: skip
+    if (lane == 0 && err) atomicExch(err, 1);
+    return;
+  }
+  uint16_t* src = qkv + m * row_stride + (long long)slot * HD;  // q | k | v heads are contiguous
+  float x[E];
+#pragma unroll
+  for (int j = 0; j < E; ++j) x[j] = bf2f(src[lane + 32 * j]);
+  const bool is_v = slot >= H + Hkv;
+  if (!is_v) {
+    const float* c = cs + (long long)p * HD;  // [p][HD/2][2]
+#pragma unroll
+    for (int j = 0; j < E / 2; ++j) {
+      const int i = lane + 32 * j;
+      const float co = c[2 * i], si = c[2 * i + 1];
+      const float a = x[j], bb = x[j + E / 2];
+      x[j] = a * co - bb * si;
+      x[j + E / 2] = bb * co + a * si;
+    }
+#pragma unroll
+    for (int j = 0; j < E; ++j) x[j] = bf2f(f2bf(x[j]));
+  }
+  if (slot < H) {
+#pragma unroll
+    for (int j = 0; j < E; ++j) src[lane + 32 * j] = f2bf(x[j]);
+    return;
+  }
+  const int kvh = is_v ? slot - H - Hkv : slot - H;
+  const int page = kv.page_table[(long long)b * kv.pages_per_seq + lp];
+  if (page < 0 || page >= kv.n_pages) {
+    if (lane == 0 && err) atomicExch(err, 1);
+    return;
+  }
+  const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + (p % kv.page_size);
+  if (KVQ == FP_KV_BF16) {
+    uint16_t* dst = (uint16_t*)(is_v ? kv.v_pool : kv.k_pool) + rowi * HD;
+#pragma unroll
+    for (int j = 0; j < E; ++j) dst[lane + 32 * j] = f2bf(x[j]);
+  } else {
+    float amax = 0.f;
+#pragma unroll
+    for (int j = 0; j < E; ++j) amax = fmaxf(amax, fabsf(x[j]));
+    amax = warp_max(amax);
+    const float sc = __fdiv_rn(amax, 127.0f);
+    int8_t* dst = (int8_t*)(is_v ? kv.v_pool : kv.k_pool) + rowi * HD;
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      float r = sc > 0.f ? rintf(__fdiv_rn(x[j], sc)) : 0.f;
+      dst[lane + 32 * j] = (int8_t)(int)fminf(fmaxf(r, -127.f), 127.f);
+    }
+    if (lane == 0) (is_v ? kv.v_scale : kv.k_scale)[rowi] = sc;
+  }
+}
+
+cudaError_t launch_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_heads, const fp_kv_view& kv,
+                           const int32_t* pos, const float* rope_cs, int32_t* err, cudaStream_t s) {
+  long long warps = (long long)B * S * (n_heads + 2 * kv.n_kv_heads);
+  if (warps <= 0) return cudaSuccess;
+  int blocks = (int)((warps + 7) / 8);
+  if (kv.head_dim == 64) {
+    if (kv.kvquant == FP_KV_BF16)
+      rope_kv_kernel<64, FP_KV_BF16><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+    else
+      rope_kv_kernel<64, FP_KV_INT8><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+  } else {
+    if (kv.kvquant == FP_KV_BF16)
+      rope_kv_kernel<128, FP_KV_BF16><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+    else
+      rope_kv_kernel<128, FP_KV_INT8><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+  }
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ positions
+__global__ void advance_kernel(int32_t* pos, int B, int by) {
+  int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) pos[b] += by;
+}
+
+cudaError_t launch_advance(int32_t* pos, int B, int by, cudaStream_t s) {
+  advance_kernel<<<(B + 127) / 128, 128, 0, s>>>(pos, B, by);
+  return cudaGetLastError();
+}
+
+}  // namespace fpk

@@ -1,0 +1,44 @@
+// Internal launchers of the fingerprint kernels.  The C entry points of
+// fp_ops.h and the runtime of fp.h both go through these; arguments are
+// validated by the callers, so the launchers only launch.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/fp_ops.h"
+
+namespace fpk {
+
+// ---- weights: seeded fill and quantisers (fp_quant.cu)
+cudaError_t launch_init_weights(uint16_t* w, long long n, unsigned long long seed, long long stream_id,
+                                long long start, cudaStream_t s);
+cudaError_t launch_quantize(int wquant, const uint16_t* w, int N, int K, void* codes, uint16_t* scales,
+                            uint16_t* zeros, cudaStream_t s);
+
+// ---- small row kernels (fp_rows.cu)
+cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h,
+                         int32_t* err, cudaStream_t s);
+cudaError_t launch_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int row_offset,
+                           const uint16_t* g, float eps, uint16_t* y, cudaStream_t s);
+cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s);
+cudaError_t launch_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_heads, const fp_kv_view& kv,
+                           const int32_t* pos, const float* rope_cs, int32_t* err, cudaStream_t s);
+cudaError_t launch_advance(int32_t* pos, int B, int by, cudaStream_t s);
+
+// ---- attention (fp_attention.cu)
+size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len);
+cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, const fp_kv_view& kv,
+                                    const int32_t* len, int len_add, int max_len, uint16_t* out, void* ws,
+                                    int32_t* err, cudaStream_t s, cudaError_t* second = nullptr);
+cudaError_t launch_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
+                                     const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s);
+
+// ---- weight-only linear (fp_linear.cu)
+size_t linear_ws_bytes(int wquant, int M, int N, int K);
+cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
+                          const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                          void* ws, cudaStream_t s);
+
+}  // namespace fpk

@@ -5,7 +5,7 @@ none of the method's arithmetic: only counter-based random draws and their
 mapping to bf16 weight values and prompt token ids.
 
 Generator (the same definition is implemented independently on the device
-in ``paper_2501_13111_gb300/csrc/fp_init.cu``):
+in ``paper_2501_13111_gb300/csrc/fp_quant.cu`` and ``common.cuh``):
 
 * SplitMix64 (Steele, Lea and Flood, OOPSLA 2014): the state advances by the
   golden-ratio increment ``GAMMA`` and each output is the state passed
@@ -93,9 +93,14 @@ def _irwin_hall_sum(u: np.ndarray) -> np.ndarray:
 
 def normal_bf16(seed: int, stream: int, start: int, count: int) -> np.ndarray:
     """bf16 bit patterns of approximately N(0, 0.02) weights (see module doc)."""
-    s = _irwin_hall_sum(draws(seed, stream, start, count))
-    v = (s - IRWIN_HALL_MEAN).astype(np.float64) * WEIGHT_SCALE_002
-    return f32_to_bf16_bits(v.astype(np.float32))
+    out = np.empty(count, dtype=np.uint16)
+    step = 1 << 20  # chunks that stay in cache
+    for lo in range(0, count, step):
+        n = min(step, count - lo)
+        s = _irwin_hall_sum(draws(seed, stream, start + lo, n))
+        v = (s - IRWIN_HALL_MEAN).astype(np.float64) * WEIGHT_SCALE_002
+        out[lo:lo + n] = f32_to_bf16_bits(v.astype(np.float32))
+    return out
 
 
 def weight_bf16(seed: int, layer: int, tensor: int, shape) -> np.ndarray:

@@ -1,0 +1,86 @@
+"""The C ABI library loads and exports every function include/*.h declares;
+host-side argument checks answer without a GPU (no compute call is made)."""
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    names = set()
+    for hdr in ("fp.h", "fp_ops.h"):
+        src = open(os.path.join(ROOT, "include", hdr)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        for m in re.finditer(r"^[A-Za-z_][\w\s\*]*?\b(fp_\w+)\s*\(", src, flags=re.M):
+            names.add(m.group(1))
+    return names
+
+
+@pytest.fixture(scope="module")
+def fp():
+    import __graft_entry__
+
+    __graft_entry__.build()
+    import paper_2501_13111_gb300 as fp
+
+    return fp
+
+
+def test_every_declared_symbol_is_exported(fp):
+    import ctypes
+
+    names = _declared()
+    assert len(names) >= 20
+    lib = ctypes.CDLL(fp.LIB_PATH)
+    for n in sorted(names):
+        assert hasattr(lib, n), n
+    # the binding covers the same names
+    assert set(fp.EXPORTED) == names
+
+
+def _arch(**kw):
+    a = dict(n_layers=1, hidden=512, n_heads=8, n_kv_heads=8, head_dim=64, ffn=1376, vocab=32000, rms_eps=1e-5,
+             rope_base=1e4)
+    a.update(kw)
+    return a
+
+
+@pytest.mark.parametrize("kw,wq,code", [
+    (dict(head_dim=96), 0, -2),
+    (dict(n_heads=8, n_kv_heads=3), 0, -1),
+    (dict(n_layers=9), 0, -2),
+    (dict(hidden=520), 0, -2),
+    (dict(ffn=1376), 2, -2),   # int4 needs ffn % 128
+    (dict(n_heads=32, n_kv_heads=2), 0, -2),  # group of 16 is not built
+    (dict(vocab=0), 0, -1),
+])
+def test_create_rejects_bad_shapes_on_host(fp, kw, wq, code):
+    with pytest.raises(fp.FPError) as e:
+        fp.fp_create(_arch(**kw), wq, 0, 1, 64)
+    assert e.value.code == code
+
+
+def test_create_rejects_bad_modes_on_host(fp):
+    for args in [(_arch(), 3, 0, 1, 64), (_arch(), 0, 2, 1, 64), (_arch(), 0, 0, 0, 64), (_arch(), 0, 0, 1, 0)]:
+        with pytest.raises(fp.FPError) as e:
+            fp.fp_create(*args)
+        assert e.value.code == fp.FP_ERR_INVALID_ARG
+    with pytest.raises(fp.FPError) as e:
+        fp.fp_create(_arch(), 0, 0, 1, 64, page_size=32)
+    assert e.value.code == fp.FP_ERR_UNSUPPORTED
+
+
+def test_op_argument_checks_on_host(fp):
+    assert fp._lib.fp_op_linear(0, 0, None, 1, 8, 8, None, None, None, None, None, None, 0, None) == -1
+    assert fp._lib.fp_op_linear(5, 0, 1, 1, 8, 8, 1, 1, 1, None, 1, None, 0, None) == -1
+    # int4 needs K % 128
+    assert fp._lib.fp_op_linear(2, 0, 1, 1, 8, 64, 1, 1, 1, None, 1, None, 0, None) == -2
+    assert fp._lib.fp_op_quantize(2, 1, 4, 100, 1, 1, 1, None) == -2
+    assert fp._lib.fp_op_rmsnorm(1, 1, 12, 1, 0, 1, 1e-5, 1, None) == -2
+    kv = fp.fp_kv_view(0, 2, 96, 16, 4, 8, 1, 1, None, None, 1)
+    assert fp.fp_op_attention_decode_workspace_bytes(2, 4, 128, 100) > 0
+    import ctypes
+    assert fp._lib.fp_op_attention_prefill(1, 1024, 1, 4, 4, ctypes.byref(kv), 1, None, None) == -2
+    assert fp.fp_strerror(-5) == "KV cache capacity exceeded"

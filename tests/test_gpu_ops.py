@@ -1,0 +1,273 @@
+"""Kernel-level parity: each entry point of fp_ops.h against the oracle on the
+same seeded inputs.  Codes, packing, ids and generated weights are compared
+bit for bit; floating-point outputs within max|d| <= tau * max|ref|."""
+import numpy as np
+import pytest
+
+import synth
+from oracle import model as M
+from oracle import quant
+from tests.gpu_helpers import TAU, dev, empty, host, ptr, rel_err, torch_mod
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def fp():
+    torch_mod()
+    import paper_2501_13111_gb300 as fp
+
+    return fp
+
+
+def _special_weights(n, k, seed):
+    w = synth.weight_bf16(seed, 2, 1, (n, k))
+    w[0] = 0
+    w[1] = 0
+    w[1, 3] = synth.f32_to_bf16_bits(np.array([0.75], np.float32))[0]
+    w[2] = synth.f32_to_bf16_bits(np.array([-0.125], np.float32))[0]
+    w[3] = synth.f32_to_bf16_bits(-np.abs(quant.bf16_to_f32(w[3])))
+    return w
+
+
+# ---------------------------------------------------------------- weights
+@pytest.mark.parametrize("seed,stream,start,n", [(0, 17, 0, 1000), (7, 3, 123456789, 4099), (2 ** 63 + 5, 99, 5, 77)])
+def test_device_generator_matches_host(fp, seed, stream, start, n):
+    w = empty(n, np.uint16)
+    fp.fp_op_init_weights(ptr(w), n, seed, stream, start)
+    assert np.array_equal(host(w, np.uint16), synth.normal_bf16(seed, stream, start, n))
+
+
+@pytest.mark.parametrize("wq,n,k", [(1, 37, 1376), (1, 256, 4096), (2, 37, 1408), (2, 130, 4096)])
+def test_quantize_bit_exact(fp, wq, n, k):
+    w = _special_weights(n, k, 5 + wq)
+    codes = empty(n * k if wq == 1 else n * k // 2)
+    scales = empty(n if wq == 1 else n * (k // 128), np.uint16)
+    zeros = empty(n * (k // 128), np.uint16)
+    fp.fp_op_quantize(wq, ptr(dev(w)), n, k, ptr(codes), ptr(scales), ptr(zeros))
+    payload, _ = quant.quantize_weight(w, wq)
+    if wq == 1:
+        assert np.array_equal(host(codes, np.int8).reshape(n, k), payload["codes"])
+        assert np.array_equal(host(scales, np.uint16), payload["scales"])
+    else:
+        assert np.array_equal(host(codes, np.uint8).reshape(n, k // 2), payload["codes"])
+        assert np.array_equal(host(scales, np.uint16).reshape(n, -1), payload["scales"])
+        assert np.array_equal(host(zeros, np.uint16).reshape(n, -1), payload["zeros"])
+
+
+# ---------------------------------------------------------------- linear
+def _quantized_on_device(fp, wq, w):
+    n, k = w.shape
+    if wq == 0:
+        return dev(w), None, None
+    codes = empty(n * k if wq == 1 else n * k // 2)
+    scales = empty(n if wq == 1 else n * (k // 128), np.uint16)
+    zeros = empty(max(1, n * (k // 128)), np.uint16)
+    fp.fp_op_quantize(wq, ptr(dev(w)), n, k, ptr(codes), ptr(scales), ptr(zeros))
+    return codes, scales, zeros
+
+
+@pytest.mark.parametrize("wq", [0, 1, 2])
+@pytest.mark.parametrize("m", [1, 3, 8, 13, 64, 130])
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_linear_matches_oracle(fp, wq, m, epi):
+    k, n = (384, 200) if wq != 2 else (512, 200)
+    w = synth.weight_bf16(11 + wq, 0, 1, (n, k))
+    x = synth.uniform_bf16(12, m, (m, k), -2.0, 2.0)
+    r = synth.uniform_bf16(13, m, (m, n), -1.0, 1.0)
+    codes, scales, zeros = _quantized_on_device(fp, wq, w)
+    _, wd = quant.quantize_weight(w, wq)
+    xf = quant.bf16_to_f32(x).astype(np.float64)
+    yref = xf @ wd.T
+    nout = n // 2 if epi == 2 else n
+    out = empty(m * nout * (4 if epi == 3 else 2))
+    rd = dev(r)
+    ws_b = fp.fp_op_linear_workspace_bytes(wq, m, n, k)
+    ws = empty(max(ws_b, 16))
+    fp.fp_op_linear(wq, epi, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(rd), ptr(out),
+                    ptr(ws), ws_b)
+    if epi == 0:
+        got, ref = host(out, np.uint16), yref
+        got = quant.bf16_to_f32(got).reshape(m, n)
+    elif epi == 1:
+        got = quant.bf16_to_f32(host(out, np.uint16)).reshape(m, n)
+        ref = quant.bf16_to_f32(r).astype(np.float64) + yref
+    elif epi == 2:
+        got = quant.bf16_to_f32(host(out, np.uint16)).reshape(m, nout)
+        ref = M.silu(yref[:, :nout]) * yref[:, nout:]
+    else:
+        got = host(out, np.float32).reshape(m, n)
+        ref = yref
+    assert rel_err(got, ref) <= TAU[wq] / 4, (wq, m, epi, rel_err(got, ref))
+
+
+def test_linear_residual_in_place(fp):
+    m, n, k = 5, 64, 256
+    w = synth.weight_bf16(3, 0, 1, (n, k))
+    x = synth.uniform_bf16(4, 1, (m, k), -1, 1)
+    r = synth.uniform_bf16(4, 2, (m, n), -1, 1)
+    codes, scales, zeros = _quantized_on_device(fp, 1, w)
+    buf = dev(r)
+    fp.fp_op_linear(1, 1, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(buf), ptr(buf), None, 0)
+    _, wd = quant.quantize_weight(w, 1)
+    ref = quant.bf16_to_f32(r) + quant.bf16_to_f32(x).astype(np.float64) @ wd.T
+    assert rel_err(quant.bf16_to_f32(host(buf, np.uint16)).reshape(m, n), ref) < 5e-3
+
+
+# ---------------------------------------------------------------- rows
+@pytest.mark.parametrize("m,d,stride,offset", [(1, 512, 1, 0), (7, 4096, 1, 0), (3, 1024, 5, 4)])
+def test_rmsnorm(fp, m, d, stride, offset):
+    rows = m * stride
+    x = synth.uniform_bf16(21, d, (rows, d), -3, 3)
+    g = synth.uniform_bf16(22, d, (d,), 0.5, 1.5)
+    y = empty(m * d, np.uint16)
+    fp.fp_op_rmsnorm(ptr(dev(x)), m, d, stride, offset, ptr(dev(g)), 1e-5, ptr(y))
+    xs = quant.bf16_to_f32(x).astype(np.float64)[offset::stride][:m]
+    ref = M.rmsnorm(xs, quant.bf16_to_f32(g).astype(np.float64), 1e-5)
+    assert rel_err(quant.bf16_to_f32(host(y, np.uint16)).reshape(m, d), ref) < 1e-2
+
+
+def test_embed_and_bad_id(fp):
+    V, d = 100, 64
+    E = synth.weight_bf16(1, -1, 0, (V, d))
+    tok = np.array([5, 0, 99, 100, -1, 7], np.int32)
+    h = empty(len(tok) * d, np.uint16)
+    err = empty(1, np.int32)
+    fp.fp_op_embed(ptr(dev(tok)), len(tok), ptr(dev(E)), V, d, ptr(h), ptr(err))
+    out = host(h, np.uint16).reshape(len(tok), d)
+    for i, t in enumerate(tok):
+        assert np.array_equal(out[i], E[t] if 0 <= t < V else np.zeros(d, np.uint16))
+    assert host(err, np.int32)[0] == 1
+
+
+@pytest.mark.parametrize("V", [32000, 17, 1000])
+def test_argmax_ties_lowest(fp, V):
+    rng = np.random.default_rng(V)
+    x = rng.normal(size=(4, V)).astype(np.float32)
+    x[1, :] = 1.0
+    x[2, [V // 3, V // 2, V - 1]] = 50.0
+    x[3, V - 1] = 60.0
+    out = empty(4, np.int32)
+    fp.fp_op_argmax(ptr(dev(x)), 4, V, ptr(out))
+    assert host(out, np.int32).tolist() == M.argmax(x.astype(np.float64)).tolist()
+
+
+# ---------------------------------------------------------------- KV cache
+class Cache:
+    """A paged cache built on the host (values chosen by the test), uploaded."""
+
+    def __init__(self, fp, kvq, B, T, Hkv, hd, seed, shuffle=True):
+        self.P, self.pps = 16, (T + 15) // 16
+        self.n_pages = B * self.pps
+        rng = np.random.default_rng(seed)
+        perm = rng.permutation(self.n_pages) if shuffle else np.arange(self.n_pages)
+        self.table = perm.reshape(B, self.pps).astype(np.int32)
+        shape = (self.n_pages, Hkv, self.P, hd)
+        self.kvq, self.B, self.Hkv, self.hd = kvq, B, Hkv, hd
+        if kvq == 0:
+            self.k = synth.uniform_bf16(seed, 1, shape, -2, 2)
+            self.v = synth.uniform_bf16(seed, 2, shape, -2, 2)
+            self.kd, self.vd = dev(self.k), dev(self.v)
+            self.ks = self.vs = None
+        else:
+            self.k = rng.integers(-127, 128, size=shape, dtype=np.int8)
+            self.v = rng.integers(-127, 128, size=shape, dtype=np.int8)
+            self.ksc = synth.uniform_f32(seed, 3, shape[:3], 0.001, 0.03)
+            self.vsc = synth.uniform_f32(seed, 4, shape[:3], 0.001, 0.03)
+            self.kd, self.vd = dev(self.k), dev(self.v)
+            self.ks, self.vs = dev(self.ksc), dev(self.vsc)
+        self.td = dev(self.table)
+        self.view = fp.fp_kv_view(kvq, Hkv, hd, self.P, self.pps, self.n_pages, ptr(self.kd), ptr(self.vd),
+                                  ptr(self.ks), ptr(self.vs), ptr(self.td))
+
+    def seq(self, which, b, T):
+        """Dequantised K or V of sequence b, positions 0..T-1: [T, Hkv, hd] fp64."""
+        pages = self.table[b, np.arange(T) // 16]
+        slot = np.arange(T) % 16
+        if self.kvq == 0:
+            src = self.k if which == "k" else self.v
+            return quant.bf16_to_f32(src[pages, :, slot]).astype(np.float64)
+        codes = (self.k if which == "k" else self.v)[pages, :, slot].astype(np.float64)
+        sc = (self.ksc if which == "k" else self.vsc)[pages, :, slot].astype(np.float64)
+        return codes * sc[..., None]
+
+
+@pytest.mark.parametrize("kvq", [0, 1])
+@pytest.mark.parametrize("hd,H,Hkv", [(64, 8, 8), (128, 8, 1), (128, 64, 8), (128, 4, 2)])
+@pytest.mark.parametrize("lens", [[1], [17, 300, 16], [1037, 5]])
+def test_attention_decode(fp, kvq, hd, H, Hkv, lens):
+    B, T = len(lens), max(lens) + 3
+    c = Cache(fp, kvq, B, T, Hkv, hd, seed=hd + H + kvq)
+    q = synth.uniform_bf16(31, B, (B, H * hd), -2, 2)
+    out = empty(B * H * hd, np.uint16)
+    wsb = fp.fp_op_attention_decode_workspace_bytes(B, H, hd, T)
+    ws = empty(wsb)
+    err = empty(1, np.int32)
+    fp.fp_op_attention_decode(ptr(dev(q)), H * hd, B, H, c.view, ptr(dev(np.array(lens, np.int32))), T, ptr(out),
+                              ptr(ws), wsb, ptr(err))
+    got = quant.bf16_to_f32(host(out, np.uint16)).reshape(B, H, hd)
+    qf = quant.bf16_to_f32(q).astype(np.float64).reshape(B, H, hd)
+    for b, L in enumerate(lens):
+        ref = M.attention(qf[b][None], np.array([L - 1]), c.seq("k", b, L), c.seq("v", b, L))[0]
+        assert rel_err(got[b], ref) <= TAU[0] / 2, (b, rel_err(got[b], ref))
+    assert host(err, np.int32)[0] == 0
+
+
+@pytest.mark.parametrize("kvq", [0, 1])
+@pytest.mark.parametrize("hd,H,Hkv", [(64, 4, 4), (128, 8, 2)])
+@pytest.mark.parametrize("S", [1, 17, 64, 130])
+def test_attention_prefill(fp, kvq, hd, H, Hkv, S):
+    B = 2
+    c = Cache(fp, kvq, B, S + 5, Hkv, hd, seed=S + hd + kvq)
+    q = synth.uniform_bf16(41, S, (B * S, H * hd), -2, 2)
+    out = empty(B * S * H * hd, np.uint16)
+    fp.fp_op_attention_prefill(ptr(dev(q)), H * hd, B, S, H, c.view, ptr(out))
+    got = quant.bf16_to_f32(host(out, np.uint16)).reshape(B, S, H, hd)
+    qf = quant.bf16_to_f32(q).astype(np.float64).reshape(B, S, H, hd)
+    for b in range(B):
+        ref = M.attention(qf[b], np.arange(S), c.seq("k", b, S), c.seq("v", b, S))
+        assert rel_err(got[b], ref) <= TAU[0] / 2, (b, rel_err(got[b], ref))
+
+
+@pytest.mark.parametrize("kvq", [0, 1])
+@pytest.mark.parametrize("hd", [64, 128])
+def test_rope_kv_write(fp, kvq, hd):
+    B, S, H, Hkv, T = 3, 5, 4, 2, 48
+    c = Cache(fp, kvq, B, T, Hkv, hd, seed=7)
+    base = 10000.0
+    cs = empty(T * hd, np.float32)
+    fp.fp_op_rope_table(T, hd, base, ptr(cs))
+    row = (H + 2 * Hkv) * hd
+    qkv = synth.uniform_bf16(51, hd, (B * S, row), -3, 3)
+    pos = np.array([0, 9, 30], np.int32)
+    qd = dev(qkv)
+    err = empty(1, np.int32)
+    fp.fp_op_rope_kv(ptr(qd), B, S, row, H, c.view, ptr(dev(pos)), ptr(cs), ptr(err))
+    q_out = quant.bf16_to_f32(host(qd, np.uint16)).reshape(B, S, -1)
+    x = quant.bf16_to_f32(qkv).astype(np.float64).reshape(B, S, H + 2 * Hkv, hd)
+    kd = host(c.kd, np.int8 if kvq else np.uint16)
+    vd = host(c.vd, np.int8 if kvq else np.uint16)
+    for b in range(B):
+        p = pos[b] + np.arange(S)
+        qref = M.rope(x[b, :, :H][None], p, base)[0]
+        assert rel_err(q_out[b, :, : H * hd].reshape(S, H, hd), qref) < 1e-2
+        kref = M.rope(x[b, :, H:H + Hkv][None], p, base)[0]
+        vref = x[b, :, H + Hkv:]
+        pages, slot = c.table[b, p // 16], p % 16
+        if kvq == 0:
+            kg = quant.bf16_to_f32(kd.reshape(c.n_pages, Hkv, 16, hd)[pages, :, slot]).astype(np.float64)
+            vg = quant.bf16_to_f32(vd.reshape(c.n_pages, Hkv, 16, hd)[pages, :, slot]).astype(np.float64)
+            assert rel_err(kg, kref) < 1e-2 and np.array_equal(vg, vref)
+        else:
+            ks = host(c.ks, np.float32).reshape(c.n_pages, Hkv, 16)[pages, :, slot]
+            vs = host(c.vs, np.float32).reshape(c.n_pages, Hkv, 16)[pages, :, slot]
+            kg = kd.reshape(c.n_pages, Hkv, 16, hd)[pages, :, slot]
+            vg = vd.reshape(c.n_pages, Hkv, 16, hd)[pages, :, slot]
+            # values: bit-exact codes (V has no rotation; K at position 0 is unrotated)
+            vq, vsr = quant.quantize_kv_int8(qkv.reshape(B, S, H + 2 * Hkv, hd)[b, :, H + Hkv:])
+            assert np.array_equal(vg, vq) and np.array_equal(vs, vsr)
+            if pos[b] == 0:
+                kq, ksr = quant.quantize_kv_int8(qkv.reshape(B, S, H + 2 * Hkv, hd)[b, 0:1, H:H + Hkv])
+                assert np.array_equal(kg[0:1], kq) and np.array_equal(ks[0:1], ksr)
+            assert rel_err(kg * ks[..., None].astype(np.float64), kref) < 1.5e-2
+    assert host(err, np.int32)[0] == 0
