@@ -116,6 +116,31 @@ int fp_op_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, 
                            size_t workspace_bytes, int32_t* err, void* stream);
 size_t fp_op_attention_decode_workspace_bytes(int B, int n_heads, int head_dim, int max_len);
 
+/* Decode attention without a caller workspace, for callers that cannot
+ * allocate device memory (a host whose device memory is all reserved by
+ * another framework's pool, a plugin that must not call the allocator, a
+ * latency-critical loop that cannot risk the synchronisation of cudaMalloc).
+ * The paper has no counterpart: this is a deployment convenience of this
+ * library only.
+ *
+ * Same arguments, kernels and results as fp_op_attention_decode, but the
+ * split partials go to a scratch array of FP_NOALLOC_SCRATCH_BYTES (32 MiB)
+ * compiled into the library.  Every GPU that loads the library holds that
+ * array until the process exits.  The call allocates nothing.
+ *   - A request whose fp_op_attention_decode_workspace_bytes(B, n_heads,
+ *     head_dim, max_len) exceeds FP_NOALLOC_SCRATCH_BYTES returns
+ *     FP_ERR_UNSUPPORTED before anything is launched.
+ *   - The first call on a device looks up the array's device address on that
+ *     device (cudaGetSymbolAddress, with the device current) and caches it;
+ *     make that first call before any stream capture.
+ *   - All calls share the one array, which keeps the last call's contents;
+ *     each call writes every partial it reads back, so nothing needs
+ *     clearing.  Calls that overlap on the GPU (other streams, other host
+ *     threads) race on the array: serialise them. */
+#define FP_NOALLOC_SCRATCH_BYTES (32u << 20)
+int fp_op_attention_decode_noalloc(const uint16_t* q, int q_stride, int B, int n_heads, const fp_kv_view* kv,
+                                   const int32_t* len, int max_len, uint16_t* out, int32_t* err, void* stream);
+
 /* Prefill attention: causal, S query rows per sequence at positions 0..S-1,
  * q bf16 [B*S][q_stride]; keys/values read from the cache positions 0..S-1;
  * out bf16 [B*S][n_heads*head_dim]. */

@@ -131,6 +131,7 @@ _PROTOS = {
     "fp_op_rope_kv": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P, _P]),
     "fp_op_attention_decode": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _SZ, _P, _P]),
     "fp_op_attention_decode_workspace_bytes": (_SZ, [_I, _I, _I, _I]),
+    "fp_op_attention_decode_noalloc": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _P]),
     "fp_op_attention_prefill": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P]),
     "fp_op_argmax": (_I, [_P, _I, _I, _P, _P]),
 }
@@ -297,6 +298,16 @@ def fp_op_attention_decode(q, q_stride, B, n_heads, kv: fp_kv_view, lens, max_le
                            workspace_bytes, err=None, stream=None):
     return _check(_lib.fp_op_attention_decode(q, q_stride, B, n_heads, C.byref(kv), lens, max_len, out, workspace,
                                               workspace_bytes, err, stream))
+
+
+FP_NOALLOC_SCRATCH_BYTES = 32 << 20
+
+
+def fp_op_attention_decode_noalloc(q, q_stride, B, n_heads, kv: fp_kv_view, lens, max_len, out, err=None,
+                                   stream=None):
+    """Decode attention with the library's own fixed scratch (no workspace argument)."""
+    return _check(_lib.fp_op_attention_decode_noalloc(q, q_stride, B, n_heads, C.byref(kv), lens, max_len, out,
+                                                      err, stream))
 
 
 def fp_op_attention_prefill(q, q_stride, B, S, n_heads, kv: fp_kv_view, out, err=None, stream=None):
