@@ -18,7 +18,10 @@ int4 weights, asymmetric, groups of 128 along K (row n, group g):
     z  = clamp(rint(fp32(-mn / s)), 0, 15)     (stored as bf16, exact)
     q  = clamp(rint(fp32(w / s)) + z, 0, 15)
     dequantised weight = (q - z) * s;  a zero range gives s = z = q = 0.
-    Packing: bytes [N][K/2]; element 2j in the low nibble, 2j+1 in the high.
+    Packing: bytes [N][K/2].  Each little-endian 32-bit word holds 8
+    consecutive elements e0..e7 of a row; nibble i (bits 4i .. 4i+3) holds
+    element NIBBLE_ORDER[i] = (0, 2, 4, 6, 1, 3, 5, 7).  So the nibble pair
+    (i, i + 4) -- the pair a mask of 0x000F000F selects -- is (e_2i, e_2i+1).
 
 int8 KV cache, per token and per KV head, separately for K (after RoPE) and V:
     s = fp32(max |x| / 127) (stored as fp32), q = clamp(rint(fp32(x / s)), -127, 127)
@@ -32,6 +35,7 @@ from __future__ import annotations
 import numpy as np
 
 GROUP = 128
+NIBBLE_ORDER = (0, 2, 4, 6, 1, 3, 5, 7)
 
 
 def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
@@ -95,17 +99,26 @@ def quantize_int4_g128(w_bits: np.ndarray):
     # the zero point is an integer in [0, 15]; "+ 0" turns rint(-0.0) into +0
     z = np.clip(np.rint(zr), 0, 15) + np.float32(0.0)
     q = np.clip(np.rint(r) + z[..., None], 0, 15).astype(np.uint8).reshape(n, k)
-    packed = (q[:, 0::2] | (q[:, 1::2] << np.uint8(4))).astype(np.uint8)
-    return packed, f32_to_bf16_rne(s), f32_to_bf16_rne(z.astype(np.float32))
+    return pack_int4(q), f32_to_bf16_rne(s), f32_to_bf16_rne(z.astype(np.float32))
+
+
+def pack_int4(q: np.ndarray) -> np.ndarray:
+    """[N, K] codes 0..15 -> [N, K/2] bytes in the nibble order above."""
+    n, k = q.shape
+    nib = q.reshape(n, k // 8, 8)[..., list(NIBBLE_ORDER)]       # nibble i <- element ORDER[i]
+    return (nib[..., 0::2] | (nib[..., 1::2] << np.uint8(4))).astype(np.uint8).reshape(n, k // 2)
 
 
 def unpack_int4(packed: np.ndarray) -> np.ndarray:
-    """[N, K/2] bytes -> [N, K] codes 0..15 (low nibble = even element)."""
+    """[N, K/2] bytes -> [N, K] codes 0..15 (inverse of pack_int4)."""
     n, kh = packed.shape
-    q = np.empty((n, kh * 2), dtype=np.uint8)
-    q[:, 0::2] = packed & np.uint8(0x0F)
-    q[:, 1::2] = packed >> np.uint8(4)
-    return q
+    b = packed.reshape(n, kh // 4, 4)
+    nib = np.empty((n, kh // 4, 8), dtype=np.uint8)
+    nib[..., 0::2] = b & np.uint8(0x0F)
+    nib[..., 1::2] = b >> np.uint8(4)
+    q = np.empty_like(nib)
+    q[..., list(NIBBLE_ORDER)] = nib
+    return q.reshape(n, kh * 2)
 
 
 def dequant_int4(packed, scale_bits, zero_bits) -> np.ndarray:

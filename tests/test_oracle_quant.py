@@ -96,7 +96,7 @@ def test_int4_hand_example():
     assert int(s[0, 0]) == g["scale_bits"]
     assert int(z[0, 0]) == g["zero_bits"]
     assert p[0, :4].tolist() == g["first_bytes"]
-    assert np.all(p[0, 2:] == 0x55)
+    assert np.all(p[0, 4:] == 0x55)
     deq = quant.dequant_int4(p, s, z)
     assert deq[0, :4].tolist() == g["dequant_first"]
 
@@ -126,10 +126,18 @@ def test_int4_codes_nearest_and_bounded():
 def test_int4_packing_order_and_roundtrip():
     rng = np.random.default_rng(0)
     q = rng.integers(0, 16, size=(3, 256), dtype=np.uint8)
-    packed = (q[:, 0::2] | (q[:, 1::2] << 4)).astype(np.uint8)
+    packed = quant.pack_int4(q)
+    assert packed.shape == (3, 128)
     assert np.array_equal(quant.unpack_int4(packed), q)
-    # element 2j sits in the low nibble of byte j
-    assert int(packed[0, 0] & 0xF) == int(q[0, 0]) and int(packed[0, 0] >> 4) == int(q[0, 1])
+    # word w of a row holds elements 8w .. 8w+7; nibble i holds element (0,2,4,6,1,3,5,7)[i]
+    word = packed[1, 4:8].astype(np.uint32)
+    word = int(word[0] | (word[1] << 8) | (word[2] << 16) | (word[3] << 24))
+    for i, e in enumerate((0, 2, 4, 6, 1, 3, 5, 7)):
+        assert (word >> (4 * i)) & 0xF == q[1, 8 + e]
+    # the 0x000F000F mask of the word shifted by 4s picks elements 2s and 2s+1
+    for s_ in range(4):
+        pair = (word >> (4 * s_)) & 0x000F000F
+        assert (pair & 0xF, pair >> 16) == (q[1, 8 + 2 * s_], q[1, 8 + 2 * s_ + 1])
 
 
 def test_int4_scale_covers_range():
