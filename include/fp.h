@@ -46,7 +46,10 @@ extern "C" {
  *   FP_W_BF16       : bf16 [N][K]
  *   FP_W_INT8       : int8 codes [N][K] + one bf16 scale per output row [N];
  *                     w = q * s, s = bf16 round-up of max|w_row| / 127
- *   FP_W_INT4_G128  : uint8 [N][K/2] (element 2j in the low nibble of byte j)
+ *   FP_W_INT4_G128  : uint8 [N][K/2]: each little-endian 32-bit word holds
+ *                     8 consecutive elements e0..e7 of a row, nibble i
+ *                     (bits 4i..4i+3) = element (0,2,4,6,1,3,5,7)[i], so the
+ *                     nibbles a 0x000F000F mask picks are a consecutive pair;
  *                     + bf16 scale and bf16 zero per row and 128-wide group
  *                     of K, [N][K/128] each; w = (q - z) * s               */
 enum { FP_W_BF16 = 0, FP_W_INT8 = 1, FP_W_INT4_G128 = 2 };

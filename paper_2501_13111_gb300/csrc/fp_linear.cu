@@ -2,23 +2,33 @@
 // y = x W^T, x bf16 [M][K], W bf16 / int8 per-channel / int4 group-128 (the
 // INT8 and INT4 weight-only configurations, Sec. 3.2; formats in fp.h).
 //
-// This file holds the memory-bound decode GEMV: a warp owns one output row
-// (two for SwiGLU: gate row n and up row n + N/2), streams the row's codes
-// with 16-byte non-allocating loads, dequantises in registers and reduces
-// over the warp; up to MT rows of x share each weight load.
+// Two kernels, chosen by the number of rows M of x:
+//  * gemv_mma_kernel (M <= 64, decode): HBM-bound.  Each warp streams 16-row
+//    tiles of codes with 16-byte non-allocating loads, turns them into bf16
+//    MMA operands in registers (raw int8 codes, 128 + int4 codes), and runs
+//    mma.sync m16n8k16 against x staged once per CTA in shared memory.
+//    Scales are applied in fp32 (int8: per row in the epilogue; int4: per
+//    128-group, s * (acc - (128 + z) * sum x)), so the weights enter exactly.
+//    K is split across CTAs; the last CTA of a row block to finish sums the
+//    partials and runs the epilogue (no spinning).
+//  * gemv_kernel (fallback: larger M or a K that is not a multiple of the
+//    MMA super-step): CUDA cores, one warp per output row.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
 namespace fpk {
 
+// Elements of K in one 16-byte chunk of codes.
 template <int WQ>
 struct WFmt;
 template <>
-struct WFmt<FP_W_BF16> { static constexpr int VE = 8;  static constexpr int RB = 2; };  // elements / 16 B chunk, row bytes per 1 element x RB/2
+struct WFmt<FP_W_BF16> { static constexpr int VE = 8; };
 template <>
-struct WFmt<FP_W_INT8> { static constexpr int VE = 16; static constexpr int RB = 1; };
+struct WFmt<FP_W_INT8> { static constexpr int VE = 16; };
 template <>
-struct WFmt<FP_W_INT4_G128> { static constexpr int VE = 32; static constexpr int RB = 0; };
+struct WFmt<FP_W_INT4_G128> { static constexpr int VE = 32; };
 
 // Row pointer of the codes of output row n.
 template <int WQ>
@@ -63,12 +73,12 @@ FP_DEV float chunk_dot(const uint4& w, const uint16_t* xp, float zero) {
     for (int h = 0; h < 4; ++h) {
       uint4 x = ld_nc16(xv + h);
       const uint32_t xx[4] = {x.x, x.y, x.z, x.w};
-      const uint32_t word = ww[h];  // 8 nibbles = elements 8h .. 8h+7
+      const uint32_t word = ww[h];  // elements 8h .. 8h+7; nibbles i and i+4 hold elements 2i and 2i+1
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         float2 b = bf2x2f(xx[i]);
-        const float lo = (float)((word >> (8 * i)) & 0xF) - zero;
-        const float hi = (float)((word >> (8 * i + 4)) & 0xF) - zero;
+        const float lo = (float)((word >> (4 * i)) & 0xF) - zero;
+        const float hi = (float)((word >> (4 * i + 16)) & 0xF) - zero;
         acc += lo * b.x + hi * b.y;
       }
     }
@@ -171,16 +181,376 @@ static cudaError_t launch_gemv(int epi, const uint16_t* x, int M, int N, int K, 
   return launch_gemv_mt<WQ, 8>(epi, x, M, N, K, codes, scales, zeros, R, y, s);
 }
 
+
+// =====================================================================
+// Decode GEMV on tensor cores (mma.sync m16n8k16, bf16 operands, fp32 acc)
+// =====================================================================
+// Thread (g = lane / 4, t = lane % 4) of a warp loads one 16-byte chunk of
+// codes per row and super-step: KT consecutive k starting at t * KT.  Its
+// k-slots of MMA k-step j are its local elements 4j .. 4j+3 (slots 2t, 2t+1
+// <- 4j, 4j+1 and slots 2t+8, 2t+9 <- 4j+2, 4j+3); x uses the same map, so
+// the contraction is unchanged.
+template <int WQ>
+struct MmaFmt;
+template <>
+struct MmaFmt<FP_W_BF16> { static constexpr int KT = 8; };
+template <>
+struct MmaFmt<FP_W_INT8> { static constexpr int KT = 16; };
+template <>
+struct MmaFmt<FP_W_INT4_G128> { static constexpr int KT = 32; };
+
+constexpr int kGemvWarps = 4;
+
+FP_DEV void mma16816(float* c, uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+FP_DEV uint32_t word_of(const uint4& w, int i) { return i == 0 ? w.x : i == 1 ? w.y : i == 2 ? w.z : w.w; }
+
+// Thread-local elements 4j + 2h, 4j + 2h + 1 of a code chunk as a bf16 pair:
+// bf16 weights as they are, int8 codes exactly, int4 as 128 + q (exact).
+template <int WQ>
+FP_DEV uint32_t apair(const uint4& w, int j, int h) {
+  if constexpr (WQ == FP_W_BF16) {
+    return word_of(w, 2 * j + h);
+  } else if constexpr (WQ == FP_W_INT8) {
+    const uint32_t word = word_of(w, j);
+    const int sh = 16 * h;
+    return pack_bf2((float)(int8_t)(word >> sh), (float)(int8_t)(word >> (sh + 8)));
+  } else {
+    // word j/2 holds elements 8(j/2) .. +7; nibbles i, i+4 hold elements 2i, 2i+1
+    const uint32_t word = word_of(w, j >> 1);
+    const int sh = 8 * (j & 1) + 4 * h;
+    return ((word >> sh) & 0x000F000Fu) | 0x43004300u;  // bf16 128 + q, low and high half
+  }
+}
+
+template <int WQ>
+FP_DEV long long code_bytes(long long k) {
+  return WQ == FP_W_BF16 ? 2 * k : WQ == FP_W_INT8 ? k : k / 2;
+}
+
+template <int WQ, int NT, int RT, int EPI>
+__global__ void __launch_bounds__(128) gemv_mma_kernel(const uint16_t* __restrict__ X, int M, int N, int K,
+                                                       const void* __restrict__ codes,
+                                                       const uint16_t* __restrict__ scales,
+                                                       const uint16_t* __restrict__ zeros, const uint16_t* R,
+                                                       void* Y, int ksplit, int splits, float* __restrict__ ws,
+                                                       unsigned* __restrict__ counters) {
+  constexpr int KT = MmaFmt<WQ>::KT, SUP = 4 * KT, KS = KT / 4, CH = KT / 8;
+  constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
+  constexpr int RTT = RT * NR;
+  extern __shared__ uint4 xs[];  // x of [kb, ke) in fragment order, then (int4) per-group row sums
+  __shared__ int s_last;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+  const int Nout = NR == 2 ? N / 2 : N;
+  const int kb = blockIdx.y * ksplit;
+  const int nsup = (min(K, kb + ksplit) - kb) / SUP;
+
+  // ---- stage x rows 0 .. 8 NT - 1 (zero at and past M):
+  //      16-byte unit ((s NT + nt) CH + c) 32 + lane <- x[nt 8 + g][kb + s SUP + t KT + 8c .. +7]
+  const int units = nsup * NT * CH * 32;
+  for (int u = threadIdx.x; u < units; u += blockDim.x) {
+    const int ln = u & 31, rest = u >> 5;
+    const int c = rest % CH, snt = rest / CH, nt = snt % NT, s = snt / NT;
+    const int m = nt * 8 + (ln >> 2);
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (m < M) v = ld_nc16(X + (long long)m * K + kb + s * SUP + (ln & 3) * KT + 8 * c);
+    xs[u] = v;
+  }
+  float* xsum = reinterpret_cast<float*>(xs + units);  // int4: [nsup][8 NT], sum of x over each group
+  __syncthreads();
+  if constexpr (WQ == FP_W_INT4_G128) {
+    for (int e = threadIdx.x; e < nsup * NT * 8; e += blockDim.x) {
+      const int s = e / (NT * 8), m = e % (NT * 8), nt = m / 8, gg = m % 8;
+      float sum = 0.f;
+#pragma unroll
+      for (int tt = 0; tt < 4; ++tt)
+#pragma unroll
+        for (int c = 0; c < CH; ++c) {
+          const uint4 v = xs[((s * NT + nt) * CH + c) * 32 + gg * 4 + tt];
+          const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = bf2x2f(w4[i]);
+            sum += f.x + f.y;
+          }
+        }
+      xsum[e] = sum;
+    }
+    __syncthreads();
+  }
+
+  // ---- this warp's rows: tile rt covers rows (tile0 + rt) * 16 + g (+8); part r: gate / up
+  const int tile0 = (blockIdx.x * kGemvWarps + warp) * RT;
+  const uint8_t* wp[RTT][2];
+  int rows[RTT][2];
+#pragma unroll
+  for (int rt = 0; rt < RT; ++rt)
+#pragma unroll
+    for (int r = 0; r < NR; ++r)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int row = (tile0 + rt) * 16 + g + 8 * h;
+        const int rc = min(row, Nout - 1) + r * Nout;
+        rows[rt * NR + r][h] = rc;
+        wp[rt * NR + r][h] = (const uint8_t*)codes + code_bytes<WQ>((long long)rc * K + kb + t * KT);
+      }
+  const int groups = K / 128;
+
+  float acc[RTT][NT][4];
+#pragma unroll
+  for (int a = 0; a < RTT; ++a)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) acc[a][nt][0] = acc[a][nt][1] = acc[a][nt][2] = acc[a][nt][3] = 0.f;
+
+  uint4 wcur[RTT][2], wnxt[RTT][2];
+  if (nsup > 0) {
+#pragma unroll
+    for (int a = 0; a < RTT; ++a) {
+      wcur[a][0] = ld_stream16(wp[a][0]);
+      wcur[a][1] = ld_stream16(wp[a][1]);
+    }
+  }
+  for (int s = 0; s < nsup; ++s) {
+    if (s + 1 < nsup) {
+#pragma unroll
+      for (int a = 0; a < RTT; ++a) {
+        wnxt[a][0] = ld_stream16(wp[a][0] + (s + 1) * 64);
+        wnxt[a][1] = ld_stream16(wp[a][1] + (s + 1) * 64);
+      }
+    }
+    float tmp[WQ == FP_W_INT4_G128 ? RTT : 1][NT][4];
+    if constexpr (WQ == FP_W_INT4_G128) {
+#pragma unroll
+      for (int a = 0; a < RTT; ++a)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) tmp[a][nt][0] = tmp[a][nt][1] = tmp[a][nt][2] = tmp[a][nt][3] = 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < KS; ++j) {
+      uint32_t b0[NT], b1[NT];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        const uint4 xv = xs[((s * NT + nt) * CH + (j >> 1)) * 32 + lane];
+        b0[nt] = (j & 1) ? xv.z : xv.x;
+        b1[nt] = (j & 1) ? xv.w : xv.y;
+      }
+#pragma unroll
+      for (int a = 0; a < RTT; ++a) {
+        const uint32_t a0 = apair<WQ>(wcur[a][0], j, 0), a1 = apair<WQ>(wcur[a][1], j, 0);
+        const uint32_t a2 = apair<WQ>(wcur[a][0], j, 1), a3 = apair<WQ>(wcur[a][1], j, 1);
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          if constexpr (WQ == FP_W_INT4_G128) mma16816(tmp[a][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
+          else mma16816(acc[a][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
+        }
+      }
+    }
+    if constexpr (WQ == FP_W_INT4_G128) {
+      // fold the group: acc += s * (sum (128 + q) x - (128 + z) sum x)
+      const int gi = (kb + s * SUP) / 128;
+#pragma unroll
+      for (int a = 0; a < RTT; ++a)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const long long si = (long long)rows[a][h] * groups + gi;
+          const float sc = bf2f(scales[si]);
+          const float zc = 128.f + bf2f(zeros[si]);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+              const float xsm = xsum[s * NT * 8 + nt * 8 + 2 * t + c];
+              acc[a][nt][2 * h + c] += sc * (tmp[a][nt][2 * h + c] - zc * xsm);
+            }
+        }
+    }
+    if (s + 1 < nsup) {
+#pragma unroll
+      for (int a = 0; a < RTT; ++a) {
+        wcur[a][0] = wnxt[a][0];
+        wcur[a][1] = wnxt[a][1];
+      }
+    }
+  }
+
+  // ---- epilogue
+  auto finish = [&](int m, int row, float v, float u) {
+    if constexpr (WQ == FP_W_INT8) {
+      v *= bf2f(scales[row]);
+      if (NR == 2) u *= bf2f(scales[row + Nout]);
+    }
+    const long long o = (long long)m * Nout + row;
+    if constexpr (EPI == FP_EPI_STORE) ((uint16_t*)Y)[o] = f2bf(v);
+    else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(bf2f(R[o]) + v);
+    else if constexpr (EPI == FP_EPI_SWIGLU) ((uint16_t*)Y)[o] = f2bf(silu(v) * u);
+    else ((float*)Y)[o] = v;
+  };
+  if (splits == 1) {
+#pragma unroll
+    for (int rt = 0; rt < RT; ++rt)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int row = (tile0 + rt) * 16 + g + 8 * (i >> 1);
+          const int m = nt * 8 + 2 * t + (i & 1);
+          if (row < Nout && m < M) finish(m, row, acc[rt * NR][nt][i], acc[rt * NR + NR - 1][nt][i]);
+        }
+    return;
+  }
+  // split-K: publish the partial, the last CTA of this row block reduces
+#pragma unroll
+  for (int rt = 0; rt < RT; ++rt)
+#pragma unroll
+    for (int r = 0; r < NR; ++r)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int row = (tile0 + rt) * 16 + g + 8 * (i >> 1);
+          const int m = nt * 8 + 2 * t + (i & 1);
+          if (row < Nout && m < M) ws[((long long)blockIdx.y * M + m) * N + row + r * Nout] = acc[rt * NR + r][nt][i];
+        }
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = atomicAdd(&counters[blockIdx.x], 1u) == (unsigned)(splits - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int rows_cta = kGemvWarps * RT * 16;
+  const int r0 = blockIdx.x * rows_cta;
+  for (int idx = threadIdx.x; idx < M * rows_cta; idx += blockDim.x) {
+    const int m = idx / rows_cta, row = r0 + idx % rows_cta;
+    if (row >= Nout) continue;
+    float v = 0.f, u = 0.f;
+    for (int sp = 0; sp < splits; ++sp) {
+      const float* p = ws + ((long long)sp * M + m) * N + row;
+      v += __ldcg(p);
+      if (NR == 2) u += __ldcg(p + Nout);
+    }
+    finish(m, row, v, u);
+  }
+  if (threadIdx.x == 0) counters[blockIdx.x] = 0u;
+}
+
+// ---------------------------------------------------------------- planning
+struct GemvPlan {
+  int NT, RT, ksplit, splits, blocks;
+  size_t smem, ws;
+};
+
+static int mma_kt(int wq) { return wq == FP_W_BF16 ? 8 : wq == FP_W_INT8 ? 16 : 32; }
+
+// Workspace = a fixed area of split-K ticket counters (zero at rest), then the
+// fp32 partials.  The ticket area has the same size for every launch, so the
+// partials of one launch never land on the counters of the next.
+constexpr int kTicketSlots = 4096;
+static size_t counter_bytes(int) { return (size_t)kTicketSlots * 4; }
+
+// Rows per CTA are at least 64, so N <= 64 * kTicketSlots keeps one ticket per row block.
+static bool mma_ok(int wq, int M, int N, int K) {
+  return M >= 1 && M <= 64 && K % (4 * mma_kt(wq)) == 0 && N <= 64 * kTicketSlots;
+}
+
+static GemvPlan plan_gemv(int wq, int epi, int M, int N, int K) {
+  GemvPlan p{};
+  const int SUP = 4 * mma_kt(wq);
+  p.NT = M <= 8 ? 1 : M <= 16 ? 2 : M <= 32 ? 4 : 8;
+  p.RT = p.NT >= 8 ? 1 : 2;
+  const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
+  if (nr == 2 && p.NT >= 4) p.RT = 1;
+  const int Nout = nr == 2 ? N / 2 : N;
+  p.blocks = (Nout + kGemvWarps * p.RT * 16 - 1) / (kGemvWarps * p.RT * 16);
+  // x chunk in shared memory: at most 64 KiB per CTA
+  const int kmax = std::max(SUP, (64 * 1024 / (p.NT * 8 * 2)) / SUP * SUP);
+  const int target = 152 * 4;
+  const int want = std::max(1, (target + p.blocks - 1) / p.blocks);
+  int ks = (K + want - 1) / want;
+  ks = (ks + SUP - 1) / SUP * SUP;
+  ks = std::min(std::max(ks, SUP), kmax);
+  p.ksplit = ks;
+  p.splits = (K + ks - 1) / ks;
+  const int nsup = ks / SUP;
+  p.smem = (size_t)nsup * p.NT * mma_kt(wq) * 64 + (wq == FP_W_INT4_G128 ? (size_t)nsup * p.NT * 8 * 4 : 0);
+  p.ws = p.splits > 1 ? counter_bytes(p.blocks) + (size_t)p.splits * M * N * 4 : 0;
+  return p;
+}
+
+template <int WQ, int NT, int RT, int EPI>
+static cudaError_t launch_mma_t(const GemvPlan& p, const uint16_t* x, int M, int N, int K, const void* codes,
+                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
+                                cudaStream_t s) {
+  auto kern = gemv_mma_kernel<WQ, NT, RT, EPI>;
+  if (p.smem > 48 * 1024)
+    FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem));
+  unsigned* counters = (unsigned*)ws;
+  float* part = ws ? (float*)((char*)ws + counter_bytes(p.blocks)) : nullptr;
+  dim3 grid(p.blocks, p.splits);
+  kern<<<grid, kGemvWarps * 32, p.smem, s>>>(x, M, N, K, codes, scales, zeros, R, y, p.ksplit, p.splits, part,
+                                             counters);
+  return cudaGetLastError();
+}
+
+template <int WQ, int EPI>
+static cudaError_t launch_mma_e(const GemvPlan& p, const uint16_t* x, int M, int N, int K, const void* codes,
+                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
+                                cudaStream_t s) {
+#define FP_MMA_CASE(nt, rt) \
+  if (p.NT == nt && p.RT == rt) return launch_mma_t<WQ, nt, rt, EPI>(p, x, M, N, K, codes, scales, zeros, R, y, ws, s);
+  FP_MMA_CASE(1, 2)
+  FP_MMA_CASE(2, 2)
+  FP_MMA_CASE(4, 2)
+  FP_MMA_CASE(4, 1)
+  FP_MMA_CASE(8, 1)
+#undef FP_MMA_CASE
+  return cudaErrorInvalidValue;
+}
+
+template <int WQ>
+static cudaError_t launch_mma(int epi, const GemvPlan& p, const uint16_t* x, int M, int N, int K, const void* codes,
+                              const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
+                              cudaStream_t s) {
+  switch (epi) {
+    case FP_EPI_STORE: return launch_mma_e<WQ, FP_EPI_STORE>(p, x, M, N, K, codes, scales, zeros, R, y, ws, s);
+    case FP_EPI_RESID: return launch_mma_e<WQ, FP_EPI_RESID>(p, x, M, N, K, codes, scales, zeros, R, y, ws, s);
+    case FP_EPI_SWIGLU: return launch_mma_e<WQ, FP_EPI_SWIGLU>(p, x, M, N, K, codes, scales, zeros, R, y, ws, s);
+    default: return launch_mma_e<WQ, FP_EPI_F32>(p, x, M, N, K, codes, scales, zeros, R, y, ws, s);
+  }
+}
+
 size_t linear_ws_bytes(int wquant, int M, int N, int K) {
-  (void)wquant; (void)M; (void)N; (void)K;
-  return 0;
+  if (!mma_ok(wquant, M, N, K)) return 0;
+  size_t a = plan_gemv(wquant, FP_EPI_STORE, M, N, K).ws;
+  size_t b = N % 2 == 0 ? plan_gemv(wquant, FP_EPI_SWIGLU, M, N, K).ws : 0;
+  return std::max(a, b);
+}
+
+size_t linear_ws_bytes_upto(int wquant, int max_m, int N, int K) {
+  size_t w = 0;
+  for (int m = 1; m <= std::min(max_m, 64); ++m) w = std::max(w, linear_ws_bytes(wquant, m, N, K));
+  return w;
 }
 
 cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
-                          void* ws, cudaStream_t s) {
-  (void)ws;
+                          void* ws, size_t ws_bytes, cudaStream_t s) {
   if (M <= 0 || N <= 0) return cudaSuccess;
+  if (mma_ok(wquant, M, N, K)) {
+    const GemvPlan p = plan_gemv(wquant, epi, M, N, K);
+    // never launch with less workspace than this plan writes
+    if (p.ws > 0 && (!ws || ws_bytes < p.ws)) return cudaErrorInvalidValue;
+    switch (wquant) {
+      case FP_W_BF16: return launch_mma<FP_W_BF16>(epi, p, x, M, N, K, codes, scales, zeros, residual, y, ws, s);
+      case FP_W_INT8: return launch_mma<FP_W_INT8>(epi, p, x, M, N, K, codes, scales, zeros, residual, y, ws, s);
+      default: return launch_mma<FP_W_INT4_G128>(epi, p, x, M, N, K, codes, scales, zeros, residual, y, ws, s);
+    }
+  }
   switch (wquant) {
     case FP_W_BF16: return launch_gemv<FP_W_BF16>(epi, x, M, N, K, codes, scales, zeros, residual, y, s);
     case FP_W_INT8: return launch_gemv<FP_W_INT8>(epi, x, M, N, K, codes, scales, zeros, residual, y, s);

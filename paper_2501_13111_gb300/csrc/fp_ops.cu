@@ -63,7 +63,7 @@ int fp_op_linear(int wquant, int epilogue, const uint16_t* x, int M, int N, int 
   size_t need = linear_ws_bytes(wquant, M, N, K);
   if (need > 0 && (!workspace || workspace_bytes < need)) return FP_ERR_INVALID_ARG;
   return cuda_status(launch_linear(wquant, epilogue, x, M, N, K, codes, scales, zeros, residual, y, workspace,
-                                   (cudaStream_t)stream));
+                                   workspace_bytes, (cudaStream_t)stream));
 }
 
 int fp_op_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int row_offset, const uint16_t* g, float eps,

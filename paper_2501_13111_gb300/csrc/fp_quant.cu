@@ -104,8 +104,14 @@ __global__ void quantize_int4_kernel(const uint16_t* __restrict__ w, int N, int 
     float r = sc > 0.f ? __fadd_rn(rintf(__fdiv_rn(v[i], sc)), z) : 0.f;
     c[i] = (uint32_t)fminf(fmaxf(r, 0.f), 15.f);
   }
-  uint16_t packed = (uint16_t)(c[0] | (c[1] << 4) | (c[2] << 8) | (c[3] << 12));
-  *reinterpret_cast<uint16_t*>(q + row * (K / 2) + g * 64 + lane * 2) = packed;
+  // Word w of the group holds elements 8w .. 8w+7 (lanes 2w and 2w+1); nibble
+  // i holds element (0,2,4,6,1,3,5,7)[i], i.e. element e sits in nibble
+  // (e >> 1) + 4 (e & 1).
+  const bool odd = lane & 1;
+  const uint32_t part = odd ? ((c[0] << 8) | (c[2] << 12) | (c[1] << 24) | (c[3] << 28))
+                            : (c[0] | (c[2] << 4) | (c[1] << 16) | (c[3] << 20));
+  const uint32_t word = part | __shfl_xor_sync(0xffffffffu, part, 1);
+  if (!odd) *reinterpret_cast<uint32_t*>(q + row * (K / 2) + g * 64 + (lane >> 1) * 4) = word;
   if (lane == 0) {
     scales[row * groups + g] = sb;
     zeros[row * groups + g] = f2bf(z);

@@ -36,9 +36,12 @@ cudaError_t launch_attention_prefill(const uint16_t* q, int q_stride, int B, int
                                      const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s);
 
 // ---- weight-only linear (fp_linear.cu)
+// Workspace of one launch with exactly these M, N, K (any epilogue); 0 if none.
 size_t linear_ws_bytes(int wquant, int M, int N, int K);
+// Largest workspace over every M in [1, max_m].
+size_t linear_ws_bytes_upto(int wquant, int max_m, int N, int K);
 cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
-                          void* ws, cudaStream_t s);
+                          void* ws, size_t ws_bytes, cudaStream_t s);
 
 }  // namespace fpk

@@ -108,7 +108,9 @@ def test_linear_residual_in_place(fp):
     r = synth.uniform_bf16(4, 2, (m, n), -1, 1)
     codes, scales, zeros = _quantized_on_device(fp, 1, w)
     buf = dev(r)
-    fp.fp_op_linear(1, 1, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(buf), ptr(buf), None, 0)
+    wsb = fp.fp_op_linear_workspace_bytes(1, m, n, k)
+    ws = empty(max(wsb, 16))
+    fp.fp_op_linear(1, 1, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(buf), ptr(buf), ptr(ws), wsb)
     _, wd = quant.quantize_weight(w, 1)
     ref = quant.bf16_to_f32(r) + quant.bf16_to_f32(x).astype(np.float64) @ wd.T
     assert rel_err(quant.bf16_to_f32(host(buf, np.uint16)).reshape(m, n), ref) < 5e-3
@@ -271,3 +273,22 @@ def test_rope_kv_write(fp, kvq, hd):
                 assert np.array_equal(kg[0:1], kq) and np.array_equal(ks[0:1], ksr)
             assert rel_err(kg * ks[..., None].astype(np.float64), kref) < 1.5e-2
     assert host(err, np.int32)[0] == 0
+
+
+def test_linear_workspace_shared_by_different_shapes(fp):
+    """One workspace serves consecutive launches of different shapes: the
+    split-K tickets left by one launch must not disturb the next."""
+    shapes = [(1, 8, 256, 4096), (1, 8, 12800, 512), (0, 1, 32000, 512), (2, 16, 2048, 1024)]
+    need = max(fp.fp_op_linear_workspace_bytes(wq, m, n, k) for wq, m, n, k in shapes)
+    ws = empty(need)
+    for rep in range(2):
+        for i, (wq, m, n, k) in enumerate(shapes):
+            w = synth.weight_bf16(40 + i, 0, 1, (n, k))
+            x = synth.uniform_bf16(41 + i, m, (m, k), -2, 2)
+            codes, scales, zeros = _quantized_on_device(fp, wq, w)
+            out = empty(m * n * 4)
+            fp.fp_op_linear(wq, 3, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), None, ptr(out),
+                            ptr(ws), need)
+            _, wd = quant.quantize_weight(w, wq)
+            ref = quant.bf16_to_f32(x).astype(np.float64) @ wd.T
+            assert rel_err(host(out, np.float32).reshape(m, n), ref) <= TAU[wq] / 4, (rep, i)
