@@ -70,6 +70,36 @@ FP_DEV uint4 ld_nc16(const void* p) { return __ldg(reinterpret_cast<const uint4*
 
 FP_DEV float silu(float x) { return x / (1.0f + __expf(-x)); }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialisation may start while the previous kernel in the stream is still
+// running.  pdl_trigger() lets the next kernel be scheduled; pdl_wait()
+// blocks until the previous kernel has completed and its writes are visible
+// (a no-op when the kernel was launched without the attribute).  Every
+// kernel of the forward pass waits before it touches activations, caches or
+// workspaces; only reads of the constant weights may come before the wait.
+FP_DEV void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+FP_DEV void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Set by the runtime while it enqueues a forward pass: launches then carry
+// the programmatic-serialisation attribute.
+extern thread_local bool g_pdl;
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                          Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = g_pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 // SplitMix64 finaliser (Steele, Lea and Flood, OOPSLA 2014).  The generator's
 // state advances by kGamma; output i of a stream keyed by K is
 // mix64(K + (i + 1) * kGamma), so draws are counter-based.

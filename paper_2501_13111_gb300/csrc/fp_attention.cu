@@ -54,6 +54,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __rest
                                                           int len_add, int max_len, int chunk, int splits,
                                                           float* __restrict__ ws, int32_t* err) {
   extern __shared__ float smem[];
+  pdl_trigger();
+  pdl_wait();
   float* sq = smem;                // [G][HD], pre-scaled by log2(e) / sqrt(hd)
   float* sp = sq + G * HD;         // [G][chunk] scores, then probabilities
   float* sml = sp + G * chunk;     // [G][2]
@@ -210,6 +212,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __rest
 template <int HD>
 __global__ void attn_combine_kernel(int H, const int32_t* __restrict__ len, int len_add, int max_len, int chunk,
                                     int splits, const float* __restrict__ ws, uint16_t* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const int bh = blockIdx.x;
   const int b = bh / H;
   const int n = (min(len[b] + len_add, max_len) + chunk - 1) / chunk;
@@ -235,11 +239,11 @@ static cudaError_t launch_decode_t(const uint16_t* q, int q_stride, int B, int H
   auto kern = attn_decode_kernel<HD, KVQ, G>;
   if (smem > 48 * 1024) FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   dim3 grid(B * kv.n_kv_heads, g.splits);
-  kern<<<grid, 128, smem, s>>>(q, q_stride, H, kv, len, len_add, max_len, g.chunk, g.splits, ws, err);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch(kern, grid, dim3(128), smem, s, q, q_stride, H, kv, len, len_add, max_len, g.chunk,
+                         g.splits, ws, err);
   if (e != cudaSuccess) return e;
-  attn_combine_kernel<HD><<<B * H, HD, 0, s>>>(H, len, len_add, max_len, g.chunk, g.splits, ws, out);
-  e = cudaGetLastError();
+  e = launch(attn_combine_kernel<HD>, dim3(B * H), dim3(HD), 0, s, H, len, len_add, max_len, g.chunk, g.splits,
+             (const float*)ws, out);
   if (second) *second = e;
   return e;
 }
@@ -312,6 +316,8 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __res
   constexpr int BT = 64;        // rows per tile
   constexpr int LD = HD + 8;    // padded row (bf16 elements) against ldmatrix bank conflicts
   extern __shared__ __align__(16) uint8_t smem_raw[];
+  pdl_trigger();
+  pdl_wait();
   uint16_t* sQ = reinterpret_cast<uint16_t*>(smem_raw);
   uint16_t* sK = sQ + BT * LD;
   uint16_t* sV = sK + BT * LD;
@@ -500,8 +506,7 @@ static cudaError_t launch_prefill_t(const uint16_t* q, int q_stride, int B, int 
   auto kern = attn_prefill_kernel<HD, KVQ>;
   if (smem > 48 * 1024) FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   dim3 grid((S + 63) / 64, H, B);
-  kern<<<grid, 128, smem, s>>>(q, q_stride, S, H, kv, out, err);
-  return cudaGetLastError();
+  return launch(kern, grid, dim3(128), smem, s, q, q_stride, S, H, kv, out, err);
 }
 
 cudaError_t launch_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,

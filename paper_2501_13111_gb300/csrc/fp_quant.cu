@@ -33,8 +33,7 @@ cudaError_t launch_init_weights(uint16_t* w, long long n, unsigned long long see
   uint64_t key = stream_key((uint64_t)seed, (uint64_t)stream_id);
   int blocks = (int)((n + 255) / 256);
   if (blocks > 152 * 16) blocks = 152 * 16;
-  init_weights_kernel<<<blocks, 256, 0, s>>>(w, n, key, start);
-  return cudaGetLastError();
+  return launch(init_weights_kernel, dim3(blocks), dim3(256), 0, s, w, n, key, start);
 }
 
 // ------------------------------------------------------------------ int8 rows
@@ -125,13 +124,11 @@ cudaError_t launch_quantize(int wquant, const uint16_t* w, int N, int K, void* c
     return cudaMemcpyAsync(codes, w, (size_t)N * K * 2, cudaMemcpyDeviceToDevice, s);
   }
   if (wquant == FP_W_INT8) {
-    quantize_int8_kernel<<<N, 256, 0, s>>>(w, K, (int8_t*)codes, scales);
-    return cudaGetLastError();
+    return launch(quantize_int8_kernel, dim3(N), dim3(256), 0, s, w, K, (int8_t*)codes, scales);
   }
   long long warps = (long long)N * (K / 128);
   int blocks = (int)((warps + 7) / 8);
-  quantize_int4_kernel<<<blocks, 256, 0, s>>>(w, N, K, (uint8_t*)codes, scales, zeros);
-  return cudaGetLastError();
+  return launch(quantize_int4_kernel, dim3(blocks), dim3(256), 0, s, w, N, K, (uint8_t*)codes, scales, zeros);
 }
 
 }  // namespace fpk

@@ -16,6 +16,8 @@ namespace fpk {
 // One CTA per token row; 16-byte copies (d % 8 == 0).
 __global__ void embed_kernel(const int32_t* __restrict__ tok, const uint16_t* __restrict__ E, int V, int d,
                              uint16_t* __restrict__ h, int32_t* err) {
+  pdl_trigger();
+  pdl_wait();
   const long long m = blockIdx.x;
   int t = tok[m];
   uint4* dst = reinterpret_cast<uint4*>(h + m * d);
@@ -32,8 +34,7 @@ __global__ void embed_kernel(const int32_t* __restrict__ tok, const uint16_t* __
 cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h, int32_t* err,
                          cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  embed_kernel<<<M, 128, 0, s>>>(tok, E, V, d, h, err);
-  return cudaGetLastError();
+  return launch(embed_kernel, dim3(M), dim3(128), 0, s, tok, E, V, d, h, err);
 }
 
 // ------------------------------------------------------------------ RMSNorm
@@ -41,6 +42,8 @@ cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, in
 // One CTA of 128 threads per row; 16-byte loads (d % 8 == 0).
 __global__ void rmsnorm_kernel(const uint16_t* __restrict__ x, int d, int row_stride, int row_offset,
                                const uint16_t* __restrict__ g, float eps, uint16_t* __restrict__ y) {
+  pdl_trigger();
+  pdl_wait();
   const long long r = blockIdx.x;
   const uint4* xr = reinterpret_cast<const uint4*>(x + ((long long)r * row_stride + row_offset) * d);
   const uint4* gr = reinterpret_cast<const uint4*>(g);
@@ -77,13 +80,14 @@ __global__ void rmsnorm_kernel(const uint16_t* __restrict__ x, int d, int row_st
 cudaError_t launch_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int row_offset, const uint16_t* g,
                            float eps, uint16_t* y, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  rmsnorm_kernel<<<M, 128, 0, s>>>(x, d, row_stride, row_offset, g, eps, y);
-  return cudaGetLastError();
+  return launch(rmsnorm_kernel, dim3(M), dim3(128), 0, s, x, d, row_stride, row_offset, g, eps, y);
 }
 
 // ------------------------------------------------------------------ argmax
 // One CTA per row; ties go to the lowest index.
 __global__ void argmax_kernel(const float* __restrict__ logits, int V, int32_t* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
   const float* lr = logits + (long long)blockIdx.x * V;
   float best = -INFINITY;
   int bi = 0x7fffffff;
@@ -118,8 +122,7 @@ __global__ void argmax_kernel(const float* __restrict__ logits, int V, int32_t* 
 
 cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  argmax_kernel<<<M, 512, 0, s>>>(logits, V, out);
-  return cudaGetLastError();
+  return launch(argmax_kernel, dim3(M), dim3(512), 0, s, logits, V, out);
 }
 
 // ------------------------------------------------------------------ RoPE + KV append
@@ -132,6 +135,8 @@ cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaS
 template <int HD, int KVQ>
 __global__ void rope_kv_kernel(uint16_t* __restrict__ qkv, int B, int S, int row_stride, int H, fp_kv_view kv,
                                const int32_t* __restrict__ pos, const float* __restrict__ cs, int32_t* err) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int E = HD / 32;
   const int Hkv = kv.n_kv_heads;
   const int slots = H + 2 * Hkv;
@@ -204,27 +209,28 @@ cudaError_t launch_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_he
   int blocks = (int)((warps + 7) / 8);
   if (kv.head_dim == 64) {
     if (kv.kvquant == FP_KV_BF16)
-      rope_kv_kernel<64, FP_KV_BF16><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+      return launch(rope_kv_kernel<64, FP_KV_BF16>, dim3(blocks), dim3(256), 0, s, qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
     else
-      rope_kv_kernel<64, FP_KV_INT8><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+      return launch(rope_kv_kernel<64, FP_KV_INT8>, dim3(blocks), dim3(256), 0, s, qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
   } else {
     if (kv.kvquant == FP_KV_BF16)
-      rope_kv_kernel<128, FP_KV_BF16><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+      return launch(rope_kv_kernel<128, FP_KV_BF16>, dim3(blocks), dim3(256), 0, s, qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
     else
-      rope_kv_kernel<128, FP_KV_INT8><<<blocks, 256, 0, s>>>(qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
+      return launch(rope_kv_kernel<128, FP_KV_INT8>, dim3(blocks), dim3(256), 0, s, qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
   }
   return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ positions
 __global__ void advance_kernel(int32_t* pos, int B, int by) {
+  pdl_trigger();
+  pdl_wait();
   int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < B) pos[b] += by;
 }
 
 cudaError_t launch_advance(int32_t* pos, int B, int by, cudaStream_t s) {
-  advance_kernel<<<(B + 127) / 128, 128, 0, s>>>(pos, B, by);
-  return cudaGetLastError();
+  return launch(advance_kernel, dim3((B + 127) / 128), dim3(128), 0, s, pos, B, by);
 }
 
 }  // namespace fpk

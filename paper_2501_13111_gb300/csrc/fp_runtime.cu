@@ -22,6 +22,10 @@ using namespace fpk;
 
 extern int fpk_check_kv(const fp_kv_view* kv);
 
+namespace fpk {
+thread_local bool g_pdl = false;
+}
+
 namespace {
 
 thread_local std::string g_create_error;
@@ -274,6 +278,11 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
   const int B = h->B, M = B * S, d = a.hidden;
   cudaStream_t s = h->stream;
   h->launches = 0;
+  // kernels of one forward overlap their start-up with the previous kernel's tail
+  struct PdlScope {
+    PdlScope() { g_pdl = true; }
+    ~PdlScope() { g_pdl = false; }
+  } pdl_scope;
   h->tr.start();
   LTRY(launch_embed(tok, M, h->embed, a.vocab, d, h->h, h->err, s), FP_K_EMBED);
   h->tr.boundary();

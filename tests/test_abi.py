@@ -84,3 +84,31 @@ def test_op_argument_checks_on_host(fp):
     import ctypes
     assert fp._lib.fp_op_attention_prefill(1, 1024, 1, 4, 4, ctypes.byref(kv), 1, None, None) == -2
     assert fp.fp_strerror(-5) == "KV cache capacity exceeded"
+
+
+def test_forward_kernels_wait_for_their_predecessor():
+    """Kernels of the forward pass are launched with programmatic dependent
+    launch, so each must execute pdl_wait() before it reads or writes
+    activations; a missing wait is a race.  Static check of the sources: every
+    __global__ kernel outside the weight set-up calls pdl_wait()."""
+    csrc = os.path.join(ROOT, "paper_2501_13111_gb300", "csrc")
+    setup_only = {"init_weights_kernel", "quantize_int8_kernel", "quantize_int4_kernel"}
+    missing = []
+    for name in os.listdir(csrc):
+        if not name.endswith(".cu"):
+            continue
+        src = open(os.path.join(csrc, name)).read()
+        for m in re.finditer(r"__global__\s+void\s+(?:__launch_bounds__\([^)]*\)\s+)?(\w+)\s*\(", src):
+            kname = m.group(1)
+            if kname in setup_only:
+                continue
+            body_start = src.index("{", m.end())
+            depth, i = 0, body_start
+            while True:
+                depth += {"{": 1, "}": -1}.get(src[i], 0)
+                if depth == 0:
+                    break
+                i += 1
+            if "pdl_wait()" not in src[body_start:i]:
+                missing.append(f"{name}:{kname}")
+    assert not missing, missing
