@@ -8,6 +8,8 @@
 // Eq. 1).  Both kernels read K and V back from the cache; with the int8 cache
 // the per-token scales multiply the scores (K) and the probabilities (V), so
 // codes enter the arithmetic exactly.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -17,49 +19,86 @@ static constexpr float kLog2e = 1.4426950408889634f;
 
 // =====================================================================
 // Decode: grid (B * Hkv, splits); one CTA handles the G = H / Hkv query
-// heads of one KV head over one chunk of the context.
+// heads of one KV head over one chunk of the context.  The chunk's K and V
+// stream through a ring of 32-token tiles in shared memory (cp.async, two
+// tiles in flight); each warp takes 8 tokens of a tile and keeps its own
+// online softmax, and the 4 warps are merged at the end.
 // =====================================================================
+constexpr int kDecTile = 32;  // tokens per tile: two 16-token pages
+constexpr int kDecBuf = 3;    // ring depth
+constexpr int kDecOcc = 4;    // resident CTAs per SM assumed by the split geometry
+
 struct DecodeGeom {
-  int chunk;   // positions per split (multiple of 16)
+  int chunk;   // positions per split (multiple of kDecTile)
   int splits;  // ceil(max_len / chunk)
 };
 
+static int dec_sm_count() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        n <= 0)
+      n = 152;
+  }
+  return n;
+}
+
+// As many splits as fill the resident CTA slots once (whole waves), at least
+// one tile per split.  Splits never grow with n_kv_heads, so the workspace
+// sized for n_kv_heads = 1 covers every launch.
 static DecodeGeom decode_geom(int B, int n_kv_heads, int max_len) {
-  // Aim for >= 4 CTAs per SM over the 152 SMs when the context allows it.
-  long long pairs = (long long)B * n_kv_heads;
-  long long want = 152 * 4;
-  long long per = (long long)max_len * pairs / want;
-  int chunk = (int)((per + 15) / 16 * 16);
-  if (chunk < 64) chunk = 64;
-  if (chunk > 512) chunk = 512;
+  const long long pairs = (long long)B * n_kv_heads;
+  const long long slots = (long long)dec_sm_count() * kDecOcc;
+  const int tiles = (max_len + kDecTile - 1) / kDecTile;
+  int splits = (int)std::max<long long>(1, slots / pairs);
+  splits = std::min(splits, tiles);
+  const int per_tiles = (tiles + splits - 1) / splits;
   DecodeGeom g;
-  g.chunk = chunk;
-  g.splits = (max_len + chunk - 1) / chunk;
+  g.chunk = per_tiles * kDecTile;
+  g.splits = (max_len + g.chunk - 1) / g.chunk;
   return g;
 }
 
 size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len) {
-  // Heads share the geometry of the KV-head split, so the worst case over
-  // Hkv (Hkv = H gives the most splits).
   DecodeGeom g = decode_geom(B, 1, max_len);
   size_t rows = (size_t)B * n_heads * g.splits;
   return rows * (size_t)(head_dim + 2) * sizeof(float);
 }
 
+FP_DEV void dec_cp_async16(void* smem, const void* gmem) {
+  const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gmem) : "memory");
+}
+FP_DEV void dec_cp_async4(void* smem, const void* gmem) {
+  const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s), "l"(gmem) : "memory");
+}
+
+template <int HD, int KVQ>
+constexpr size_t dec_smem_bytes() {
+  return (size_t)kDecBuf * kDecTile * HD * (KVQ == FP_KV_BF16 ? 2 : 1) * 2 +
+         (KVQ == FP_KV_INT8 ? (size_t)kDecBuf * kDecTile * 2 * sizeof(float) : 0);
+}
+
 // Workspace layout for (b, h, split): o [HD] fp32 (un-normalised, relative to
-// the chunk max), then (m, l) in the log2 domain.
+// m), then (m, l) in the log2 domain.
 template <int HD, int KVQ, int G>
 __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __restrict__ q, int q_stride, int H,
                                                           fp_kv_view kv, const int32_t* __restrict__ len,
                                                           int len_add, int max_len, int chunk, int splits,
                                                           float* __restrict__ ws, int32_t* err) {
-  extern __shared__ float smem[];
+  constexpr int TT = kDecTile, NBUF = kDecBuf;
+  constexpr int ELT = KVQ == FP_KV_BF16 ? 2 : 1, ROWB = HD * ELT, TILEB = TT * ROWB, CPR = ROWB / 16;
+  constexpr int DPL = HD / 32;                   // dims per lane
+  constexpr int TG = G >= 4 ? 2 : (G == 2 ? 4 : 8);  // tokens per softmax update
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint8_t* sK = smem;                  // [NBUF][TT][ROWB]
+  uint8_t* sV = sK + NBUF * TILEB;     // [NBUF][TT][ROWB]
+  float* sKs = reinterpret_cast<float*>(sV + NBUF * TILEB);  // int8: [NBUF][TT]
+  float* sVs = sKs + NBUF * TT;
   pdl_trigger();
   pdl_wait();
-  float* sq = smem;                // [G][HD], pre-scaled by log2(e) / sqrt(hd)
-  float* sp = sq + G * HD;         // [G][chunk] scores, then probabilities
-  float* sml = sp + G * chunk;     // [G][2]
-  float* sred = sml + 2 * G;       // [4][G][HD]
   const int Hkv = kv.n_kv_heads;
   const int b = blockIdx.x / Hkv, kvh = blockIdx.x % Hkv;
   const int split = blockIdx.y;
@@ -70,140 +109,198 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __rest
   }
   const int t0 = split * chunk;
   if (t0 >= T) return;
-  const int nt = min(chunk, T - t0);
+  const int t1 = min(T, t0 + chunk);
+  const int ntile = (t1 - t0 + TT - 1) / TT;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const float qscale = kLog2e * rsqrtf((float)HD);
-  for (int i = tid; i < G * HD; i += 128) {
-    int g = i / HD, e = i % HD;
-    sq[i] = bf2f(q[(long long)b * q_stride + (long long)(kvh * G + g) * HD + e]) * qscale;
-  }
-  __syncthreads();
-
   const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
-  // ---- scores: LPT lanes per token, 16 bytes of the K row per lane
-  constexpr int ELT = KVQ == FP_KV_BF16 ? 2 : 1;
-  constexpr int EPL = 16 / ELT;
-  constexpr int LPT = HD / EPL;
-  constexpr int TPW = 32 / LPT;
-  const int sub = lane % LPT, grp = lane / LPT;
-  for (int base = warp * TPW; base < nt; base += 4 * TPW) {
-    const int ti = base + grp;
-    const bool valid = ti < nt;
-    float kf[EPL];
-    float ks = 1.f;
-    if (valid) {
-      const int t = t0 + ti;
-      const int page = pt[t / kv.page_size];
+
+  // ---- issue one tile of K, V (and their int8 scales) into ring slot tile % NBUF
+  auto issue = [&](int tile) {
+    const int tt0 = t0 + tile * TT;
+    uint8_t* dK = sK + (tile % NBUF) * TILEB;
+    uint8_t* dV = sV + (tile % NBUF) * TILEB;
+    for (int c = tid; c < TT * CPR; c += 128) {
+      const int j = c / CPR, part = c % CPR, t = tt0 + j;
+      const int lp = t / kv.page_size;
+      if (lp >= kv.pages_per_seq) continue;  // past the sequence's table: masked below
+      const int page = pt[lp];
+      uint8_t* dk = dK + j * ROWB + part * 16;
+      uint8_t* dv = dV + j * ROWB + part * 16;
       if (page < 0 || page >= kv.n_pages) {
-        if (err) atomicExch(err, 1);
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) kf[e] = 0.f;
-      } else {
+        if (err && t < t1) atomicExch(err, 1);
+        continue;
+      }
+      const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
+      dec_cp_async16(dk, (const uint8_t*)kv.k_pool + rowi * ROWB + part * 16);
+      dec_cp_async16(dv, (const uint8_t*)kv.v_pool + rowi * ROWB + part * 16);
+    }
+    if constexpr (KVQ == FP_KV_INT8) {
+      for (int j = tid; j < TT; j += 128) {
+        const int t = tt0 + j, lp = t / kv.page_size;
+        if (lp >= kv.pages_per_seq) continue;
+        const int page = pt[lp];
+        if (page < 0 || page >= kv.n_pages) continue;
         const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
-        uint4 raw = ld_stream16((const uint8_t*)kv.k_pool + rowi * HD * ELT + sub * 16);
-        uint32_t w[4] = {raw.x, raw.y, raw.z, raw.w};
-        if constexpr (KVQ == FP_KV_BF16) {
+        dec_cp_async4(sKs + (tile % NBUF) * TT + j, kv.k_scale + rowi);
+        dec_cp_async4(sVs + (tile % NBUF) * TT + j, kv.v_scale + rowi);
+      }
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            float2 f = bf2x2f(w[i]);
-            kf[2 * i] = f.x;
-            kf[2 * i + 1] = f.y;
+  for (int i = 0; i < NBUF - 1; ++i) {
+    if (i < ntile) issue(i);
+    else asm volatile("cp.async.commit_group;" ::: "memory");
+  }
+
+  // q of the G heads, this lane's dims, pre-scaled by log2(e) / sqrt(hd)
+  const float qscale = kLog2e * rsqrtf((float)HD);
+  float qr[G][DPL];
+#pragma unroll
+  for (int g = 0; g < G; ++g)
+#pragma unroll
+    for (int d = 0; d < DPL; ++d)
+      qr[g][d] = bf2f(q[(long long)b * q_stride + (long long)(kvh * G + g) * HD + lane * DPL + d]) * qscale;
+  float m[G], l[G], acc[G][DPL];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    m[g] = -INFINITY;
+    l[g] = 0.f;
+#pragma unroll
+    for (int d = 0; d < DPL; ++d) acc[g][d] = 0.f;
+  }
+
+  for (int tile = 0; tile < ntile; ++tile) {
+    asm volatile("cp.async.wait_group %0;" ::"n"(NBUF - 2) : "memory");
+    __syncthreads();  // tile landed for every thread; the slot refilled below is free
+    if (tile + NBUF - 1 < ntile) issue(tile + NBUF - 1);
+    else asm volatile("cp.async.commit_group;" ::: "memory");
+    const int slot = tile % NBUF;
+    const uint8_t* tK = sK + slot * TILEB;
+    const uint8_t* tV = sV + slot * TILEB;
+    const int tt0 = t0 + tile * TT;
+#pragma unroll
+    for (int grp = 0; grp < 8 / TG; ++grp) {
+      float sc[TG][G];
+#pragma unroll
+      for (int i = 0; i < TG; ++i) {
+        const int j = warp * 8 + grp * TG + i;
+        if (tt0 + j < t1) {  // warp-uniform
+          float kf[DPL];
+          if constexpr (KVQ == FP_KV_BF16) {
+            if constexpr (DPL == 4) {
+              const uint2 raw = *reinterpret_cast<const uint2*>(tK + j * ROWB + lane * 8);
+              const float2 a = bf2x2f(raw.x), c = bf2x2f(raw.y);
+              kf[0] = a.x; kf[1] = a.y; kf[2] = c.x; kf[3] = c.y;
+            } else {
+              const float2 a = bf2x2f(*reinterpret_cast<const uint32_t*>(tK + j * ROWB + lane * 4));
+              kf[0] = a.x; kf[1] = a.y;
+            }
+          } else {
+            uint32_t raw;
+            if constexpr (DPL == 4) raw = *reinterpret_cast<const uint32_t*>(tK + j * ROWB + lane * 4);
+            else raw = *reinterpret_cast<const uint16_t*>(tK + j * ROWB + lane * 2);
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) kf[d] = (float)(int8_t)((raw >> (8 * d)) & 0xFF);
+          }
+          const float ks = KVQ == FP_KV_INT8 ? sKs[slot * TT + j] : 1.f;
+#pragma unroll
+          for (int g = 0; g < G; ++g) {
+            float a = 0.f;
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) a += qr[g][d] * kf[d];
+            sc[i][g] = warp_sum(a) * ks;
           }
         } else {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) kf[i] = (float)(int8_t)((w[i >> 2] >> (8 * (i & 3))) & 0xFF);
-          ks = kv.k_scale[rowi];
+          for (int g = 0; g < G; ++g) sc[i][g] = -INFINITY;
         }
       }
-    } else {
+      // online softmax over these TG tokens
+      float p[TG][G];
 #pragma unroll
-      for (int e = 0; e < EPL; ++e) kf[e] = 0.f;
-    }
+      for (int g = 0; g < G; ++g) {
+        float mx = m[g];
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const float* qg = sq + g * HD + sub * EPL;
-      float acc = 0.f;
+        for (int i = 0; i < TG; ++i) mx = fmaxf(mx, sc[i][g]);
+        const float ref = mx == -INFINITY ? 0.f : mx;
+        const float corr = exp2f(m[g] - ref);
+        float ps = 0.f;
 #pragma unroll
-      for (int e = 0; e < EPL; ++e) acc += kf[e] * qg[e];
+        for (int i = 0; i < TG; ++i) {
+          p[i][g] = exp2f(sc[i][g] - ref);
+          ps += p[i][g];
+        }
+        l[g] = l[g] * corr + ps;
+        m[g] = mx;
 #pragma unroll
-      for (int o = LPT / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-      if (valid && sub == 0) sp[g * chunk + ti] = acc * ks;
-    }
-  }
-  __syncthreads();
-  // ---- softmax per head over the chunk (warp g handles heads g, g+4, ...)
-  for (int g = warp; g < G; g += 4) {
-    float m = -INFINITY;
-    for (int i = lane; i < nt; i += 32) m = fmaxf(m, sp[g * chunk + i]);
-    m = warp_max(m);
-    float l = 0.f;
-    for (int i = lane; i < nt; i += 32) {
-      float p = exp2f(sp[g * chunk + i] - m);
-      sp[g * chunk + i] = p;
-      l += p;
-    }
-    l = warp_sum(l);
-    if (lane == 0) {
-      sml[2 * g] = m;
-      sml[2 * g + 1] = l;
-    }
-  }
-  __syncthreads();
-  // ---- P V: lane holds HD/32 dims, warps split the tokens
-  constexpr int DPL = HD / 32;
-  float acc[G][DPL];
-#pragma unroll
-  for (int g = 0; g < G; ++g)
-#pragma unroll
-    for (int j = 0; j < DPL; ++j) acc[g][j] = 0.f;
-  for (int ti = warp; ti < nt; ti += 4) {
-    const int t = t0 + ti;
-    const int page = pt[t / kv.page_size];
-    if (page < 0 || page >= kv.n_pages) continue;
-    const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
-    float vf[DPL];
-    float vs = 1.f;
-    if constexpr (KVQ == FP_KV_BF16) {
-      const uint16_t* vr = (const uint16_t*)kv.v_pool + rowi * HD + lane * DPL;
-      if constexpr (DPL == 4) {
-        uint2 raw = *reinterpret_cast<const uint2*>(vr);
-        float2 a = bf2x2f(raw.x), c = bf2x2f(raw.y);
-        vf[0] = a.x; vf[1] = a.y; vf[2] = c.x; vf[3] = c.y;
-      } else {
-        float2 a = bf2x2f(*reinterpret_cast<const uint32_t*>(vr));
-        vf[0] = a.x; vf[1] = a.y;
+        for (int d = 0; d < DPL; ++d) acc[g][d] *= corr;
       }
-    } else {
-      const int8_t* vr = (const int8_t*)kv.v_pool + rowi * HD + lane * DPL;
-      uint32_t raw;
-      if constexpr (DPL == 4) raw = *reinterpret_cast<const uint32_t*>(vr);
-      else raw = *reinterpret_cast<const uint16_t*>(vr);
 #pragma unroll
-      for (int j = 0; j < DPL; ++j) vf[j] = (float)(int8_t)((raw >> (8 * j)) & 0xFF);
-      vs = kv.v_scale[rowi];
-    }
+      for (int i = 0; i < TG; ++i) {
+        const int j = warp * 8 + grp * TG + i;
+        if (tt0 + j < t1) {
+          float vf[DPL];
+          if constexpr (KVQ == FP_KV_BF16) {
+            if constexpr (DPL == 4) {
+              const uint2 raw = *reinterpret_cast<const uint2*>(tV + j * ROWB + lane * 8);
+              const float2 a = bf2x2f(raw.x), c = bf2x2f(raw.y);
+              vf[0] = a.x; vf[1] = a.y; vf[2] = c.x; vf[3] = c.y;
+            } else {
+              const float2 a = bf2x2f(*reinterpret_cast<const uint32_t*>(tV + j * ROWB + lane * 4));
+              vf[0] = a.x; vf[1] = a.y;
+            }
+          } else {
+            uint32_t raw;
+            if constexpr (DPL == 4) raw = *reinterpret_cast<const uint32_t*>(tV + j * ROWB + lane * 4);
+            else raw = *reinterpret_cast<const uint16_t*>(tV + j * ROWB + lane * 2);
+            const float vs = sVs[slot * TT + j];
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const float p = sp[g * chunk + ti] * vs;
+            for (int d = 0; d < DPL; ++d) vf[d] = (float)(int8_t)((raw >> (8 * d)) & 0xFF) * vs;
+          }
 #pragma unroll
-      for (int j = 0; j < DPL; ++j) acc[g][j] += p * vf[j];
+          for (int g = 0; g < G; ++g)
+#pragma unroll
+            for (int d = 0; d < DPL; ++d) acc[g][d] += p[i][g] * vf[d];
+        }
+      }
     }
   }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();  // the ring is reused for the merge below
+
+  // ---- merge the 4 warps: per head, o = sum_w acc_w 2^(m_w - M), l = sum_w l_w 2^(m_w - M)
+  float* red = reinterpret_cast<float*>(smem);  // [4][G][HD + 2]
 #pragma unroll
-  for (int g = 0; g < G; ++g)
+  for (int g = 0; g < G; ++g) {
+    float* r = red + (warp * G + g) * (HD + 2);
 #pragma unroll
-    for (int j = 0; j < DPL; ++j) sred[(warp * G + g) * HD + lane * DPL + j] = acc[g][j];
+    for (int d = 0; d < DPL; ++d) r[lane * DPL + d] = acc[g][d];
+    if (lane == 0) {
+      r[HD] = m[g];
+      r[HD + 1] = l[g];
+    }
+  }
   __syncthreads();
   for (int i = tid; i < G * HD; i += 128) {
     const int g = i / HD, e = i % HD;
-    float o = sred[(0 * G + g) * HD + e] + sred[(1 * G + g) * HD + e] + sred[(2 * G + g) * HD + e] +
-              sred[(3 * G + g) * HD + e];
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, red[(w * G + g) * (HD + 2) + HD]);
+    float o = 0.f, L = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float* r = red + (w * G + g) * (HD + 2);
+      const float f = r[HD] == -INFINITY ? 0.f : exp2f(r[HD] - M);
+      o += r[e] * f;
+      L += r[HD + 1] * f;
+    }
     const long long row = ((long long)b * H + kvh * G + g) * splits + split;
     float* w = ws + row * (HD + 2);
     w[e] = o;
     if (e == 0) {
-      w[HD] = sml[2 * g];
-      w[HD + 1] = sml[2 * g + 1];
+      w[HD] = M;
+      w[HD + 1] = L;
     }
   }
 }
@@ -235,7 +332,8 @@ template <int HD, int KVQ, int G>
 static cudaError_t launch_decode_t(const uint16_t* q, int q_stride, int B, int H, const fp_kv_view& kv,
                                    const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
                                    uint16_t* out, int32_t* err, cudaStream_t s, cudaError_t* second) {
-  size_t smem = ((size_t)G * HD + (size_t)G * g.chunk + 2 * G + 4 * (size_t)G * HD) * sizeof(float);
+  // the ring also holds the 4-warp merge buffer after the loop
+  const size_t smem = std::max(dec_smem_bytes<HD, KVQ>(), (size_t)4 * G * (HD + 2) * sizeof(float));
   auto kern = attn_decode_kernel<HD, KVQ, G>;
   if (smem > 48 * 1024) FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   dim3 grid(B * kv.n_kv_heads, g.splits);
