@@ -1,0 +1,386 @@
+// Prefill weight-only linear on the 5th-generation tensor cores.
+//
+// y[M][N] = x[M][K] W[N][K]^T for M > 64 (prefill), the dense contraction of
+// the block's linear layers.  A CTA computes one 128 x 256 output tile over
+// the whole K:
+//   warp 0      TMA producer: x tile [128][64] and W tile [256][64] (bf16,
+//               128-byte swizzled, K-major) into a 4-stage shared ring,
+//               completion counted in bytes on mbarrier full[s];
+//   warp 1      allocates 256 TMEM columns and, from one thread, issues
+//               tcgen05.mma (M 128, N 256, K 16, fp32 accumulation in TMEM);
+//               tcgen05.commit frees each stage (empty[s]) and finally
+//               signals the epilogue;
+//   warps 2-5   epilogue: tcgen05.ld of the accumulator (one TMEM lane per
+//               output row), per-column int8 scale, residual add / SwiGLU /
+//               fp32 store.
+// Quantised weights are first expanded to bf16 into a scratch matrix by
+// dequant_kernel (int8: the code itself, exact, with its row scale applied
+// in the epilogue; int4: bf16((q - z) * s)).
+//
+// Every mbarrier wait is bounded: past the limit the thread records an error
+// in the error word, the CTA stops issuing work and falls through to the TMEM
+// release, so a fault in the pipeline surfaces as a status, not a hang.
+#include <cuda.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.cuh"
+
+namespace fpk {
+
+constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64, kTcStages = 4;
+constexpr int kTcThreads = 192;
+constexpr uint32_t kTcStageBytes = (kTcBM + kTcBN) * kTcBK * 2;  // 48 KiB
+constexpr uint32_t kTcTmemCols = 256;
+constexpr long long kTcSpinLimit = 1LL << 20;  // try_wait rounds; legit waits here are < 1 ms
+
+// ------------------------------------------------------------------ PTX helpers
+FP_DEV uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+FP_DEV void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+FP_DEV void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+// Bounded wait for the completion of phase `parity`; false after the limit.
+FP_DEV bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  const uint32_t a = smem_u32(bar);
+  for (long long it = 0; it < kTcSpinLimit; ++it) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(done)
+        : "r"(a), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+
+FP_DEV void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (stride byte offset), fixed field 0b001 at bit 46.
+FP_DEV uint64_t sdesc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFF) >> 4);
+  d |= (uint64_t)1 << 16;              // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;    // stride byte offset
+  d |= (uint64_t)1 << 46;              // fixed 0b001
+  d |= (uint64_t)2 << 61;              // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, both
+// K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+constexpr uint32_t tc_idesc(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+FP_DEV void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+FP_DEV void tc_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+FP_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+FP_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+FP_DEV void tc_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+      "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// ------------------------------------------------------------------ kernel
+// SCALE: multiply output column n by bf16 scales[n] (int8 weights).
+template <int EPI, bool SCALE>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int M, int N,
+                   int K, const uint16_t* __restrict__ scales, const uint16_t* R, void* Y, int32_t* err) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ uint64_t full[kTcStages], empty[kTcStages], tmem_full;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_word;
+  volatile int* abort_flag = &abort_word;  // set by a role that gave up waiting
+  // stage buffers must be 1024-byte aligned for the 128-byte swizzle
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
+  const int Nout = NR == 2 ? N / 2 : N;
+  constexpr int BNout = kTcBN / NR;
+  const int n0 = blockIdx.x * BNout, m0 = blockIdx.y * kTcBM;
+  const int kblocks = (K + kTcBK - 1) / kTcBK;
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kTcStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(&tmem_full, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
+                 "r"(kTcTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base;
+  pdl_wait();
+
+  if (warp == 0) {
+    // ---------------- TMA producer
+    if (lane == 0) {
+      for (int kb = 0; kb < kblocks; ++kb) {
+        const int s = kb % kTcStages;
+        if (!mbar_wait(&empty[s], ((kb / kTcStages) & 1) ^ 1) || *abort_flag) {
+          *abort_flag = 1;
+          if (err) atomicExch(err, 2);
+          break;
+        }
+        uint8_t* a = smem + s * kTcStageBytes;
+        uint8_t* b = a + kTcBM * kTcBK * 2;
+        mbar_expect_tx(&full[s], kTcStageBytes);
+        tma_load_2d(a, &map_x, kb * kTcBK, m0, &full[s]);
+        if (NR == 1) {
+          tma_load_2d(b, &map_w, kb * kTcBK, n0, &full[s]);
+        } else {
+          tma_load_2d(b, &map_w, kb * kTcBK, n0, &full[s]);                              // gate rows
+          tma_load_2d(b + 128 * kTcBK * 2, &map_w, kb * kTcBK, Nout + n0, &full[s]);  // up rows
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc_idesc(kTcBM, kTcBN);
+      for (int kb = 0; kb < kblocks; ++kb) {
+        const int s = kb % kTcStages;
+        if (!mbar_wait(&full[s], (kb / kTcStages) & 1) || *abort_flag) {
+          *abort_flag = 1;
+          if (err) atomicExch(err, 2);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a = smem_u32(smem + s * kTcStageBytes);
+        const uint32_t b = a + kTcBM * kTcBK * 2;
+#pragma unroll
+        for (int kk = 0; kk < kTcBK / 16; ++kk)
+          tc_mma(tmem, sdesc(a + kk * 32), sdesc(b + kk * 32), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&empty[s]);  // stage s is free once these MMAs have read it
+      }
+      tc_commit(&tmem_full);  // all MMAs done (or none, on abort: the barrier still flips)
+    }
+  } else {
+    // ---------------- epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31
+    const int q = warp & 3;
+    const int row = m0 + q * 32 + lane;
+    const bool ok = mbar_wait(&tmem_full, 0);
+    if (!ok && err) atomicExch(err, 2);
+    tc_fence_after();
+    if (ok && !*abort_flag) {
+      const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
+#pragma unroll 1
+      for (int c0 = 0; c0 < BNout; c0 += 32) {
+        float v[32], u[32];
+        tc_ld32(tl + c0, v);
+        if (NR == 2) tc_ld32(tl + 128 + c0, u);
+        if (row >= M) continue;
+        const int n = n0 + c0;
+        if (n >= Nout) continue;
+        const int cnt = min(32, Nout - n);
+        if constexpr (SCALE) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if (i < cnt) {
+              v[i] *= bf2f(scales[n + i]);
+              if (NR == 2) u[i] *= bf2f(scales[Nout + n + i]);
+            }
+          }
+        }
+        const long long o = (long long)row * Nout + n;
+        if constexpr (EPI == FP_EPI_F32) {
+          float* y = (float*)Y + o;
+          if (cnt == 32 && (o & 3) == 0) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) *reinterpret_cast<float4*>(y + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+          } else {
+            for (int i = 0; i < cnt; ++i) y[i] = v[i];
+          }
+        } else {
+          uint16_t* y = (uint16_t*)Y + o;
+          float r[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if constexpr (EPI == FP_EPI_SWIGLU) r[i] = silu(v[i]) * u[i];
+            else r[i] = v[i];
+          }
+          if constexpr (EPI == FP_EPI_RESID) {
+            const uint16_t* rr = R + o;
+            for (int i = 0; i < cnt; ++i) r[i] += bf2f(rr[i]);
+          }
+          if (cnt == 32 && (o & 7) == 0) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 8)
+              *reinterpret_cast<uint4*>(y + i) = make_uint4(pack_bf2(r[i], r[i + 1]), pack_bf2(r[i + 2], r[i + 3]),
+                                                            pack_bf2(r[i + 4], r[i + 5]), pack_bf2(r[i + 6], r[i + 7]));
+          } else {
+            for (int i = 0; i < cnt; ++i) y[i] = f2bf(r[i]);
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols) : "memory");
+  }
+}
+
+// ------------------------------------------------------------------ dequant to bf16
+// int8: w = q (exact; the row scale is applied by the GEMM epilogue).
+// int4: w = bf16((q - z) * s), 8 elements (one packed word) per thread.
+__global__ void dequant_kernel(int wquant, const void* __restrict__ codes, const uint16_t* __restrict__ scales,
+                               const uint16_t* __restrict__ zeros, int N, int K, uint16_t* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
+  const long long words = (long long)N * K / 8;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < words; i += (long long)gridDim.x * blockDim.x) {
+    const long long e0 = i * 8;
+    const long long row = e0 / K;
+    const int k0 = (int)(e0 % K);
+    float f[8];
+    if (wquant == FP_W_INT8) {
+      const uint2 c = *reinterpret_cast<const uint2*>((const int8_t*)codes + e0);
+      const uint32_t w[2] = {c.x, c.y};
+#pragma unroll
+      for (int j = 0; j < 8; ++j) f[j] = (float)(int8_t)((w[j >> 2] >> (8 * (j & 3))) & 0xFF);
+    } else {
+      const uint32_t w = *reinterpret_cast<const uint32_t*>((const uint8_t*)codes + e0 / 2);
+      const long long gi = row * (K / 128) + k0 / 128;
+      const float s = bf2f(scales[gi]), z = bf2f(zeros[gi]);
+      // nibbles i and i + 4 hold elements 2i and 2i + 1
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        f[2 * j] = ((float)((w >> (4 * j)) & 0xF) - z) * s;
+        f[2 * j + 1] = ((float)((w >> (4 * j + 16)) & 0xF) - z) * s;
+      }
+    }
+    *reinterpret_cast<uint4*>(out + e0) =
+        make_uint4(pack_bf2(f[0], f[1]), pack_bf2(f[2], f[3]), pack_bf2(f[4], f[5]), pack_bf2(f[6], f[7]));
+  }
+}
+
+// ------------------------------------------------------------------ host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &p, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (EncodeTiledFn)p;
+  }
+  return fn;
+}
+
+// bf16 [rows][cols] row-major, box [box_rows][64] with 128-byte swizzle.
+static bool make_map(CUtensorMap* map, const void* base, long long rows, long long cols, int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {(cuuint32_t)kTcBK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t gemm_tc_ws_bytes(int wquant, int N, int K) { return wquant == FP_W_BF16 ? 0 : (size_t)N * K * 2; }
+
+bool gemm_tc_ok(int M, int N, int K) { return M > 64 && K % 8 == 0 && N >= 1 && encode_fn() != nullptr; }
+
+template <int EPI, bool SCALE>
+static cudaError_t launch_tc_t(const CUtensorMap& mx, const CUtensorMap& mw, int M, int N, int K,
+                               const uint16_t* scales, const uint16_t* R, void* Y, int32_t* err, cudaStream_t s) {
+  auto kern = gemm_tc_kernel<EPI, SCALE>;
+  const size_t smem = (size_t)kTcStages * kTcStageBytes + 1024;
+  static bool attr = false;
+  if (!attr) {
+    FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    attr = true;
+  }
+  const int Nout = EPI == FP_EPI_SWIGLU ? N / 2 : N;
+  const int bn = kTcBN / (EPI == FP_EPI_SWIGLU ? 2 : 1);
+  dim3 grid((Nout + bn - 1) / bn, (M + kTcBM - 1) / kTcBM);
+  return launch(kern, grid, dim3(kTcThreads), smem, s, mx, mw, M, N, K, scales, R, Y, err);
+}
+
+cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
+                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                           void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s) {
+  const uint16_t* w = (const uint16_t*)codes;
+  if (wquant != FP_W_BF16) {
+    if (!ws || ws_bytes < gemm_tc_ws_bytes(wquant, N, K)) return cudaErrorInvalidValue;
+    const long long words = (long long)N * K / 8;
+    const int blocks = (int)std::min<long long>((words + 255) / 256, 152 * 16);
+    FP_CUDA_TRY(launch(dequant_kernel, dim3(blocks), dim3(256), 0, s, wquant, codes, scales, zeros, N, K, (uint16_t*)ws));
+    w = (const uint16_t*)ws;
+  }
+  CUtensorMap mx, mw;
+  const int wbox = epi == FP_EPI_SWIGLU ? 128 : 256;
+  if (!make_map(&mx, x, M, K, kTcBM) || !make_map(&mw, w, N, K, wbox)) return cudaErrorInvalidValue;
+  const bool sc = wquant == FP_W_INT8;
+  switch (epi) {
+    case FP_EPI_STORE:
+      return sc ? launch_tc_t<FP_EPI_STORE, true>(mx, mw, M, N, K, scales, residual, y, err, s)
+                : launch_tc_t<FP_EPI_STORE, false>(mx, mw, M, N, K, scales, residual, y, err, s);
+    case FP_EPI_RESID:
+      return sc ? launch_tc_t<FP_EPI_RESID, true>(mx, mw, M, N, K, scales, residual, y, err, s)
+                : launch_tc_t<FP_EPI_RESID, false>(mx, mw, M, N, K, scales, residual, y, err, s);
+    case FP_EPI_SWIGLU:
+      return sc ? launch_tc_t<FP_EPI_SWIGLU, true>(mx, mw, M, N, K, scales, residual, y, err, s)
+                : launch_tc_t<FP_EPI_SWIGLU, false>(mx, mw, M, N, K, scales, residual, y, err, s);
+    default:
+      return sc ? launch_tc_t<FP_EPI_F32, true>(mx, mw, M, N, K, scales, residual, y, err, s)
+                : launch_tc_t<FP_EPI_F32, false>(mx, mw, M, N, K, scales, residual, y, err, s);
+  }
+}
+
+}  // namespace fpk

@@ -644,7 +644,14 @@ static cudaError_t launch_mma(int epi, const uint16_t* x, int M, int N, int K, c
   }
 }
 
+// Workspace of one linear launch: the ticket area, then either split-K
+// partials (decode GEMV) or the bf16 expansion of quantised weights (prefill
+// GEMM).  The ticket area is never written by the prefill path.
 size_t linear_ws_bytes(int wquant, int M, int N, int K) {
+  if (M > 64 && gemm_tc_ok(M, N, K)) {
+    const size_t w = gemm_tc_ws_bytes(wquant, N, K);
+    return w ? counter_bytes(0) + w : 0;
+  }
   if (!mma_ok(wquant, M, N, K)) return 0;
   // splits grow with occupancy, so the plan at the planner's cap (8) bounds every launch
   size_t a = plan_gemv(wquant, FP_EPI_STORE, M, N, K, 8).ws;
@@ -655,13 +662,21 @@ size_t linear_ws_bytes(int wquant, int M, int N, int K) {
 size_t linear_ws_bytes_upto(int wquant, int max_m, int N, int K) {
   size_t w = 0;
   for (int m = 1; m <= std::min(max_m, 64); ++m) w = std::max(w, linear_ws_bytes(wquant, m, N, K));
+  if (max_m > 64) w = std::max(w, linear_ws_bytes(wquant, max_m, N, K));
   return w;
 }
 
 cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
-                          void* ws, size_t ws_bytes, cudaStream_t s) {
+                          void* ws, size_t ws_bytes, cudaStream_t s, int32_t* err) {
   if (M <= 0 || N <= 0) return cudaSuccess;
+  if (M > 64 && gemm_tc_ok(M, N, K)) {
+    const size_t need = linear_ws_bytes(wquant, M, N, K);
+    if (need > 0 && (!ws || ws_bytes < need)) return cudaErrorInvalidValue;
+    void* scratch = need ? (char*)ws + counter_bytes(0) : nullptr;
+    return launch_gemm_tc(wquant, epi, x, M, N, K, codes, scales, zeros, residual, y, scratch,
+                          need ? ws_bytes - counter_bytes(0) : 0, err, s);
+  }
   if (mma_ok(wquant, M, N, K)) {
     switch (wquant) {
       case FP_W_BF16: return launch_mma<FP_W_BF16>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s);

@@ -229,7 +229,7 @@ void carve(fp_handle* h, char* base) {
   h->attn_ws = c.take<void>(h->attn_ws_bytes, &h->ws_bytes);
   // every row count a forward can use: B (decode, LM head) and B * S for any prompt S
   size_t lw = 0;
-  for (int m = 0; m < 4; ++m) lw = std::max(lw, linear_ws_bytes_upto(h->wq, (int)std::min<long long>(R, 64), NK[m][0], NK[m][1]));
+  for (int m = 0; m < 4; ++m) lw = std::max(lw, linear_ws_bytes_upto(h->wq, (int)R, NK[m][0], NK[m][1]));
   lw = std::max(lw, linear_ws_bytes_upto(FP_W_BF16, h->B, (int)V, (int)d));
   h->lin_ws_bytes = lw;
   h->lin_ws = lw ? c.take<void>(lw, &h->ws_bytes) : nullptr;
@@ -292,7 +292,7 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
     LTRY(launch_rmsnorm(h->h, M, d, 1, 0, Ly.attn_norm, a.rms_eps, h->y, s), FP_K_RMSNORM);
     const Mat& Q = Ly.mat[FP_M_QKV];
     LTRY(launch_linear(h->wq, FP_EPI_STORE, h->y, M, Q.N, Q.K, Q.codes, Q.scales, Q.zeros, nullptr, h->qkv,
-                       h->lin_ws, h->lin_ws_bytes, s),
+                       h->lin_ws, h->lin_ws_bytes, s, h->err),
          FP_K_LIN_QKV);
     LTRY(launch_rope_kv(h->qkv, B, S, h->n_qkv, a.n_heads, kv, h->pos, h->rope_cs, h->err, s), FP_K_ROPE_KV);
     if (decode) {
@@ -308,16 +308,16 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
     }
     const Mat& O = Ly.mat[FP_M_O];
     LTRY(launch_linear(h->wq, FP_EPI_RESID, h->att, M, O.N, O.K, O.codes, O.scales, O.zeros, h->h, h->h,
-                       h->lin_ws, h->lin_ws_bytes, s),
+                       h->lin_ws, h->lin_ws_bytes, s, h->err),
          FP_K_LIN_O);
     LTRY(launch_rmsnorm(h->h, M, d, 1, 0, Ly.ffn_norm, a.rms_eps, h->y, s), FP_K_RMSNORM);
     const Mat& GU = Ly.mat[FP_M_GU];
     LTRY(launch_linear(h->wq, FP_EPI_SWIGLU, h->y, M, GU.N, GU.K, GU.codes, GU.scales, GU.zeros, nullptr, h->act,
-                       h->lin_ws, h->lin_ws_bytes, s),
+                       h->lin_ws, h->lin_ws_bytes, s, h->err),
          FP_K_LIN_GU);
     const Mat& D = Ly.mat[FP_M_DOWN];
     LTRY(launch_linear(h->wq, FP_EPI_RESID, h->act, M, D.N, D.K, D.codes, D.scales, D.zeros, h->h, h->h,
-                       h->lin_ws, h->lin_ws_bytes, s),
+                       h->lin_ws, h->lin_ws_bytes, s, h->err),
          FP_K_LIN_DOWN);
     if (h->hidden) {
       cudaError_t e = cudaMemcpyAsync(h->hidden + (size_t)l * h->max_rows * d, h->h, (size_t)M * d * 2,
@@ -328,7 +328,7 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
   }
   LTRY(launch_rmsnorm(h->h, B, d, S, S - 1, h->final_norm, a.rms_eps, h->ylast, s), FP_K_RMSNORM);
   LTRY(launch_linear(FP_W_BF16, FP_EPI_F32, h->ylast, B, a.vocab, d, h->lm_head, nullptr, nullptr, nullptr,
-                     h->logits, h->lin_ws, h->lin_ws_bytes, s),
+                     h->logits, h->lin_ws, h->lin_ws_bytes, s, h->err),
        FP_K_LM_HEAD);
   LTRY(launch_argmax(h->logits, B, a.vocab, h->tokens, s), FP_K_ARGMAX);
   LTRY(launch_advance(h->pos, B, S, s), FP_K_ARGMAX);

@@ -42,6 +42,13 @@ size_t linear_ws_bytes(int wquant, int M, int N, int K);
 size_t linear_ws_bytes_upto(int wquant, int max_m, int N, int K);
 cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
-                          void* ws, size_t ws_bytes, cudaStream_t s);
+                          void* ws, size_t ws_bytes, cudaStream_t s, int32_t* err = nullptr);
+
+// ---- prefill GEMM on tcgen05 (fp_gemm_tc.cu)
+bool gemm_tc_ok(int M, int N, int K);
+size_t gemm_tc_ws_bytes(int wquant, int N, int K);
+cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
+                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                           void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s);
 
 }  // namespace fpk

@@ -292,3 +292,34 @@ def test_linear_workspace_shared_by_different_shapes(fp):
             _, wd = quant.quantize_weight(w, wq)
             ref = quant.bf16_to_f32(x).astype(np.float64) @ wd.T
             assert rel_err(host(out, np.float32).reshape(m, n), ref) <= TAU[wq] / 4, (rep, i)
+
+
+@pytest.mark.parametrize("wq", [0, 1, 2])
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+@pytest.mark.parametrize("m,n,k", [(65, 520, 1408), (300, 1024, 4096), (1000, 2304, 1024)])
+def test_prefill_gemm_matches_oracle(fp, wq, epi, m, n, k):
+    """Rows > 64 run on the tcgen05 GEMM: ragged M and N tiles, K tails."""
+    w = synth.weight_bf16(60 + wq, 0, 1, (n, k))
+    x = synth.uniform_bf16(61, m, (m, k), -2.0, 2.0)
+    r = synth.uniform_bf16(62, m, (m, n), -1.0, 1.0)
+    codes, scales, zeros = _quantized_on_device(fp, wq, w)
+    _, wd = quant.quantize_weight(w, wq)
+    yref = quant.bf16_to_f32(x).astype(np.float64) @ wd.T
+    nout = n // 2 if epi == 2 else n
+    out = empty(m * nout * (4 if epi == 3 else 2))
+    rd = dev(r[:, :nout].copy())
+    wsb = fp.fp_op_linear_workspace_bytes(wq, m, n, k)
+    ws = empty(max(wsb, 16))
+    fp.fp_op_linear(wq, epi, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(rd), ptr(out), ptr(ws), wsb)
+    if epi == 3:
+        got = host(out, np.float32).reshape(m, n)
+        ref = yref
+    else:
+        got = quant.bf16_to_f32(host(out, np.uint16)).reshape(m, nout)
+        if epi == 0:
+            ref = yref
+        elif epi == 1:
+            ref = quant.bf16_to_f32(r[:, :nout]).astype(np.float64) + yref
+        else:
+            ref = M.silu(yref[:, :nout]) * yref[:, nout:]
+    assert rel_err(got, ref) <= TAU[wq] / 4, (wq, epi, m, n, k, rel_err(got, ref))
