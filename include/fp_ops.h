@@ -55,13 +55,15 @@ enum {
 /* Weight-only linear y = x W^T (the "linear layers" of the block) with the
  * dequantisation fused: x bf16 [M][K]; W in the wquant format of fp.h
  * (codes / scales / zeros as fp_op_quantize writes them); fp32 accumulation.
- * Kernel choice depends on M and K only.  workspace: at least
+ * Kernel choice depends on M, N and K: M <= 64 runs the decode GEMV (the
+ * work is cut into equal ranges of (128-row block, K step), one per resident
+ * CTA, and shared blocks are reduced from fp32 partials in a fixed order),
+ * larger M the tcgen05 GEMM.  workspace: 16-byte aligned, at least
  * fp_op_linear_workspace_bytes(wquant, M, N, K) bytes (may be NULL when that
- * is 0), else FP_ERR_INVALID_ARG.  Its leading bytes are split-K ticket
- * counters that must be zero before the first call (e.g. a zeroed buffer);
- * every call leaves them zero again, so one workspace serves any sequence
- * of calls on one stream (calls that overlap on the GPU need separate
- * workspaces). */
+ * is 0), else FP_ERR_INVALID_ARG.  Its leading bytes are ticket counters
+ * that must be zero before the first call (e.g. a zeroed buffer); every call
+ * leaves them zero again, so one workspace serves any sequence of calls on
+ * one stream (calls that overlap on the GPU need separate workspaces). */
 int fp_op_linear(int wquant, int epilogue, const uint16_t* x, int M, int N, int K, const void* codes,
                  const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
                  void* workspace, size_t workspace_bytes, void* stream);

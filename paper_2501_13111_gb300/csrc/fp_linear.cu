@@ -9,8 +9,9 @@
 //    mma.sync m16n8k16 against x staged once per CTA in shared memory.
 //    Scales are applied in fp32 (int8: per row in the epilogue; int4: per
 //    128-group, s * (acc - (128 + z) * sum x)), so the weights enter exactly.
-//    K is split across CTAs; the last CTA of a row block to finish sums the
-//    partials and runs the epilogue (no spinning).
+//    The (row block, K step) work is cut into equal contiguous ranges, one
+//    per resident CTA; a row block shared by several CTAs is finished by the
+//    last of them from fp32 partials (no spinning).
 //  * gemv_kernel (fallback: larger M or a K that is not a multiple of the
 //    MMA super-step): CUDA cores, one warp per output row.
 #include <algorithm>
@@ -289,183 +290,89 @@ FP_DEV float2 x_pair(uint32_t w) {
   }
 }
 
-// cp.async ring depth per warp: deeper for one tile, shallower for gate + up.
-__host__ __device__ constexpr int gemv_stages(int tiles) { return tiles >= 2 ? 3 : 4; }
+// cp.async ring depth per warp (NB - 1 stages in flight): deeper for one
+// tile, shallower for gate + up.
+__host__ __device__ constexpr int gemv_stages(int tiles) { return tiles >= 2 ? 3 : 6; }
 
-template <int WQ, int NT, int RT, int EPI>
+// The work of one launch is the sequence of (row block, super-step) pairs,
+// row block major: blocks x S with S = K / super-step.  CTA c of C takes the
+// contiguous range [c total / C, (c+1) total / C), so every CTA streams the
+// same number of weight bytes whatever N and K are, and one wave of
+// resident CTAs covers the launch.  A range crosses row blocks: the CTA
+// accumulates each block's part separately and, where a block is shared by
+// several CTAs, the last to finish sums their fp32 partials in CTA order
+// (deterministic) and runs the epilogue.
+FP_DEV long long gemv_cta_of(long long i, long long C, long long total) { return ((i + 1) * C - 1) / total; }
+
+template <int WQ, int NT, int EPI>
 __global__ void __launch_bounds__(kGemvWarps * 32) gemv_mma_kernel(const uint16_t* __restrict__ X, int M, int N, int K,
                                                        const void* __restrict__ codes,
                                                        const uint16_t* __restrict__ scales,
                                                        const uint16_t* __restrict__ zeros, const uint16_t* R,
-                                                       void* Y, int ksplit, int splits, float* __restrict__ ws,
-                                                       unsigned* __restrict__ counters) {
+                                                       void* Y, long long total, int S, int W,
+                                                       float* __restrict__ ws, unsigned* __restrict__ counters) {
   constexpr int KT = MmaFmt<WQ>::KT, SUP = 4 * KT, KS = KT / 4, CH = KT / 8;
   constexpr bool F16 = WQ != FP_W_BF16;
+  constexpr bool G128 = WQ == FP_W_INT4_G128;
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
-  constexpr int RTT = RT * NR;
-  constexpr int NB = gemv_stages(RTT);  // ring stages per warp (NB - 1 in flight)
-  extern __shared__ uint4 xs[];  // x of [kb, ke) in fragment order, then fp32 column sums
+  constexpr int NB = gemv_stages(NR);
+  constexpr int ROWS = kGemvWarps * 16;  // rows of a block
+  extern __shared__ uint4 smem[];        // weight ring, then the x window, then its fp32 column sums
   __shared__ int s_last;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
   const int Nout = NR == 2 ? N / 2 : N;
-  const int kb = blockIdx.y * ksplit;
-  const int nsup = (min(K, kb + ksplit) - kb) / SUP;
+  const int groups = K / 128;
+  const long long C = gridDim.x, c = blockIdx.x;
+  const long long begin = c * total / C, end = (c + 1) * total / C;
+  const int L = (int)(end - begin);
 
-  // ---- this warp's rows: tile rt covers rows (tile0 + rt) * 16 + g (+8); part r: gate / up
-  const int tile0 = (blockIdx.x * kGemvWarps + warp) * RT;
-  const uint8_t* wp[RTT][2];
-  int rows[RTT][2];
-#pragma unroll
-  for (int rt = 0; rt < RT; ++rt)
+  uint4* ring = smem;
+  uint4* xs = smem + kGemvWarps * NB * NR * 2 * 32;
+  float* xsum = reinterpret_cast<float*>(xs + W * NT * CH * 32);
+  auto slot = [&](int stage, int r, int h) { return ring + (((warp * NB + stage) * NR + r) * 2 + h) * 32 + lane; };
+  auto row_of = [&](int blk, int h) { return blk * ROWS + warp * 16 + g + 8 * h; };
+
+  // ---- weight ring: each thread copies its own 16-byte chunks with cp.async
+  // and later reads back only those, so the ring needs no barrier.  Stage q
+  // of this CTA is super-step (begin + q) % S of row block (begin + q) / S.
+  int pf_blk = (int)(begin / S), pf_ss = (int)(begin % S);
+  const uint8_t* pw[NR][2];
+  auto set_rows = [&](int blk) {
 #pragma unroll
     for (int r = 0; r < NR; ++r)
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        const int row = (tile0 + rt) * 16 + g + 8 * h;
-        const int rc = min(row, Nout - 1) + r * Nout;
-        rows[rt * NR + r][h] = rc;
-        wp[rt * NR + r][h] = (const uint8_t*)codes + code_bytes<WQ>((long long)rc * K + kb + t * KT);
+        const int rc = min(row_of(blk, h), Nout - 1) + r * Nout;
+        pw[r][h] = (const uint8_t*)codes + code_bytes<WQ>((long long)rc * K + t * KT);
       }
+  };
+  set_rows(pf_blk);
+  auto issue = [&](int q) {  // called for q = 0, 1, 2, ... in order
+    if (q < L) {
+#pragma unroll
+      for (int r = 0; r < NR; ++r)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) cp_async16(slot(q % NB, r, h), pw[r][h] + pf_ss * 64);
+      if (++pf_ss == S) {
+        pf_ss = 0;
+        set_rows(++pf_blk);  // row pointers are clamped, so a block past the end is harmless
+      }
+    }
+    cp_async_commit();
+  };
   pdl_trigger();
-  // Weight chunks go through a per-warp ring in shared memory: each thread
-  // copies its own 16-byte chunks with cp.async and later reads back only
-  // those, so the ring needs no barrier.  The first stages go out before x
-  // is staged.
-  const int units = nsup * NT * CH * 32;
-  const int xsum_entries = WQ == FP_W_BF16 ? 0 : (WQ == FP_W_INT8 ? 1 : nsup) * NT * 8;
-  uint4* ring = xs + units + (xsum_entries + 3) / 4;
-  auto slot = [&](int stage, int a, int h) { return ring + (((warp * NB + stage) * RTT + a) * 2 + h) * 32 + lane; };
+  // weights are constant: the first stages go out before waiting on the producer of x
 #pragma unroll
-  for (int b = 0; b < NB - 1; ++b) {
-    if (b < nsup) {
-#pragma unroll
-      for (int a = 0; a < RTT; ++a) {
-        cp_async16(slot(b, a, 0), wp[a][0] + b * 64);
-        cp_async16(slot(b, a, 1), wp[a][1] + b * 64);
-      }
-    }
-    cp_async_commit();
-  }
-
-  // weights are constant; everything below reads or writes the previous kernels' data
+  for (int q = 0; q < NB - 1; ++q) issue(q);
   pdl_wait();
-  // ---- stage x rows 0 .. 8 NT - 1 (zero at and past M) as MMA operands:
-  //      16-byte unit ((s NT + nt) CH + c) 32 + lane <- x[nt 8 + g][kb + s SUP + t KT + 8c .. +7]
-  // and, for codes, the fp32 column sums of the staged operands: int8 over the
-  // CTA's K range [8 NT], int4 per super-step (= one 128-group) [nsup][8 NT].
-  float* xsum = reinterpret_cast<float*>(xs + units);
-  if constexpr (F16) {
-    for (int e = threadIdx.x; e < xsum_entries; e += blockDim.x) xsum[e] = 0.f;
-    __syncthreads();
-  }
-  // units / 32 is a whole number, so every warp iterates with all 32 lanes
-  for (int u = threadIdx.x; u < units; u += blockDim.x) {
-    const int ln = u & 31, rest = u >> 5;
-    const int c = rest % CH, snt = rest / CH, nt = snt % NT, s = snt / NT;
-    const int m = nt * 8 + (ln >> 2);
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (m < M) v = x_operand<WQ>(ld_nc16(X + (long long)m * K + kb + s * SUP + (ln & 3) * KT + 8 * c));
-    xs[u] = v;
-    if constexpr (F16) {
-      const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
-      float sum = 0.f;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float2 f = x_pair<WQ>(w4[i]);
-        sum += f.x + f.y;
-      }
-      // the 4 lanes of one x row (same g) hold consecutive pieces of it
-      sum += __shfl_xor_sync(0xffffffffu, sum, 1);
-      sum += __shfl_xor_sync(0xffffffffu, sum, 2);
-      if ((ln & 3) == 0) atomicAdd(&xsum[(WQ == FP_W_INT8 ? 0 : s * NT * 8) + m], sum);
-    }
-  }
-  __syncthreads();
-  const int groups = K / 128;
 
-  float acc[RTT][NT][4];
+  float acc[NR][NT][4];
+  auto zero_acc = [&]() {
 #pragma unroll
-  for (int a = 0; a < RTT; ++a)
+    for (int r = 0; r < NR; ++r)
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) acc[a][nt][0] = acc[a][nt][1] = acc[a][nt][2] = acc[a][nt][3] = 0.f;
-
-  for (int s = 0; s < nsup; ++s) {
-    cp_async_wait<NB - 2>();  // this thread's copies of stage s have landed
-    uint4 w[RTT][2];
-#pragma unroll
-    for (int a = 0; a < RTT; ++a) {
-      w[a][0] = *slot(s % NB, a, 0);
-      w[a][1] = *slot(s % NB, a, 1);
-    }
-    // refill the slot consumed one step ago with stage s + NB - 1
-    const int sp = s + NB - 1;
-    if (sp < nsup) {
-#pragma unroll
-      for (int a = 0; a < RTT; ++a) {
-        cp_async16(slot(sp % NB, a, 0), wp[a][0] + sp * 64);
-        cp_async16(slot(sp % NB, a, 1), wp[a][1] + sp * 64);
-      }
-    }
-    cp_async_commit();
-    float tmp[WQ == FP_W_INT4_G128 ? RTT : 1][NT][4];
-    if constexpr (WQ == FP_W_INT4_G128) {
-#pragma unroll
-      for (int a = 0; a < RTT; ++a)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) tmp[a][nt][0] = tmp[a][nt][1] = tmp[a][nt][2] = tmp[a][nt][3] = 0.f;
-    }
-#pragma unroll
-    for (int j = 0; j < KS; ++j) {
-      uint32_t b0[NT], b1[NT];
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        const uint4 xv = xs[((s * NT + nt) * CH + (j >> 1)) * 32 + lane];
-        b0[nt] = (j & 1) ? xv.z : xv.x;
-        b1[nt] = (j & 1) ? xv.w : xv.y;
-      }
-#pragma unroll
-      for (int a = 0; a < RTT; ++a) {
-        const uint32_t a0 = apair<WQ>(w[a][0], j, 0), a1 = apair<WQ>(w[a][1], j, 0);
-        const uint32_t a2 = apair<WQ>(w[a][0], j, 1), a3 = apair<WQ>(w[a][1], j, 1);
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-          if constexpr (WQ == FP_W_INT4_G128) mma16816<F16>(tmp[a][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
-          else mma16816<F16>(acc[a][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
-        }
-      }
-    }
-    if constexpr (WQ == FP_W_INT4_G128) {
-      // acc += s * (sum (1024 + q) x - (1024 + z) sum x) over the group
-      const int gi = (kb + s * SUP) / 128;
-#pragma unroll
-      for (int a = 0; a < RTT; ++a)
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const long long si = (long long)rows[a][h] * groups + gi;
-          const float sc = bf2f(scales[si]);
-          const float zc = 1024.f + bf2f(zeros[si]);
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int c = 0; c < 2; ++c) {
-              const float xsm = xsum[s * NT * 8 + nt * 8 + 2 * t + c];
-              acc[a][nt][2 * h + c] += sc * (tmp[a][nt][2 * h + c] - zc * xsm);
-            }
-        }
-    }
-  }
-  cp_async_wait<0>();
-  if constexpr (WQ == FP_W_INT8) {
-    // remove the 1152 offset of the codes: acc - 1152 * sum x over this K range
-#pragma unroll
-    for (int a = 0; a < RTT; ++a)
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) acc[a][nt][i] -= 1152.f * xsum[nt * 8 + 2 * t + (i & 1)];
-  }
-
-  // ---- epilogue
+      for (int nt = 0; nt < NT; ++nt) acc[r][nt][0] = acc[r][nt][1] = acc[r][nt][2] = acc[r][nt][3] = 0.f;
+  };
   auto finish = [&](int m, int row, float v, float u) {
     if constexpr (WQ == FP_W_INT8) {
       v *= bf2f(scales[row]);
@@ -477,71 +384,219 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_mma_kernel(const uint16_
     else if constexpr (EPI == FP_EPI_SWIGLU) ((uint16_t*)Y)[o] = f2bf(silu(v) * u);
     else ((float*)Y)[o] = v;
   };
-  if (splits == 1) {
+  zero_acc();
+
+  long long cur = begin;
+  int q = 0;
+  while (cur < end) {
+    const int b = (int)(cur / S), s0 = (int)(cur % S);
+    const long long seg_end = min(end, (long long)(b + 1) * S);
+    const int wlen = (int)min((long long)W, seg_end - cur);
+
+    // ---- stage x for super-steps s0 .. s0 + wlen - 1 of K as MMA operands:
+    //      16-byte unit ((l NT + nt) CH + c) 32 + lane <- x[nt 8 + g][(s0 + l) SUP + t KT + 8c .. +7]
+    // (zero at and past M) and, for codes, the fp32 column sums of the staged
+    // operands: int8 over the window [8 NT], int4 per super-step (= one
+    // 128-group) [wlen][8 NT].
+    const int units = wlen * NT * CH * 32;
+    const int nsum = F16 ? (G128 ? wlen : 1) * NT * 8 : 0;
+    __syncthreads();  // the previous window is consumed
+    for (int e = threadIdx.x; e < nsum; e += blockDim.x) xsum[e] = 0.f;
+    if constexpr (F16) __syncthreads();
+    constexpr int XU = 4;  // independent x loads in flight per thread
+    // units is a multiple of 32, so the lanes of a warp agree on u < units
+    for (int u0 = threadIdx.x; u0 < units; u0 += XU * blockDim.x) {
+      uint4 v[XU];
 #pragma unroll
-    for (int rt = 0; rt < RT; ++rt)
+      for (int i = 0; i < XU; ++i) {
+        const int u = u0 + i * blockDim.x;
+        const int ln = u & 31, rest = u >> 5;
+        const int cc = rest % CH, lnt = rest / CH, nt = lnt % NT, l = lnt / NT;
+        const int m = nt * 8 + (ln >> 2);
+        v[i] = make_uint4(0, 0, 0, 0);
+        if (u < units && m < M) v[i] = ld_nc16(X + (long long)m * K + (s0 + l) * SUP + (ln & 3) * KT + 8 * cc);
+      }
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
+      for (int i = 0; i < XU; ++i) {
+        const int u = u0 + i * blockDim.x;
+        if (u < units) {
+          const int ln = u & 31, rest = u >> 5;
+          const int lnt = rest / CH, nt = lnt % NT, l = lnt / NT;
+          const uint4 xo = x_operand<WQ>(v[i]);
+          xs[u] = xo;
+          if constexpr (F16) {
+            const uint32_t w4[4] = {xo.x, xo.y, xo.z, xo.w};
+            float sum = 0.f;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int row = (tile0 + rt) * 16 + g + 8 * (i >> 1);
-          const int m = nt * 8 + 2 * t + (i & 1);
-          if (row < Nout && m < M) finish(m, row, acc[rt * NR][nt][i], acc[rt * NR + NR - 1][nt][i]);
+            for (int p = 0; p < 4; ++p) {
+              const float2 f = x_pair<WQ>(w4[p]);
+              sum += f.x + f.y;
+            }
+            // the 4 lanes of one x row (same g) hold consecutive pieces of it
+            sum += __shfl_xor_sync(0xffffffffu, sum, 1);
+            sum += __shfl_xor_sync(0xffffffffu, sum, 2);
+            if ((ln & 3) == 0) atomicAdd(&xsum[(G128 ? l * NT * 8 : 0) + nt * 8 + (ln >> 2)], sum);
+          }
         }
-    return;
-  }
-  // split-K: publish the partial, the last CTA of this row block reduces
-#pragma unroll
-  for (int rt = 0; rt < RT; ++rt)
-#pragma unroll
-    for (int r = 0; r < NR; ++r)
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const int row = (tile0 + rt) * 16 + g + 8 * (i >> 1);
-          const int m = nt * 8 + 2 * t + (i & 1);
-          if (row < Nout && m < M) ws[((long long)blockIdx.y * M + m) * N + row + r * Nout] = acc[rt * NR + r][nt][i];
-        }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = atomicAdd(&counters[blockIdx.x], 1u) == (unsigned)(splits - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  const int rows_cta = kGemvWarps * RT * 16;
-  const int r0 = blockIdx.x * rows_cta;
-  for (int idx = threadIdx.x; idx < M * rows_cta; idx += blockDim.x) {
-    const int m = idx / rows_cta, row = r0 + idx % rows_cta;
-    if (row >= Nout) continue;
-    float v = 0.f, u = 0.f;
-    for (int sp = 0; sp < splits; ++sp) {
-      const float* p = ws + ((long long)sp * M + m) * N + row;
-      v += __ldcg(p);
-      if (NR == 2) u += __ldcg(p + Nout);
+      }
     }
-    finish(m, row, v, u);
+    __syncthreads();
+
+    // ---- the window's super-steps
+    for (int l = 0; l < wlen; ++l, ++q) {
+      cp_async_wait<NB - 2>();  // this thread's copies of stage q have landed
+      uint4 w[NR][2];
+#pragma unroll
+      for (int r = 0; r < NR; ++r) {
+        w[r][0] = *slot(q % NB, r, 0);
+        w[r][1] = *slot(q % NB, r, 1);
+      }
+      issue(q + NB - 1);  // refills the slot consumed one step ago
+      float sz[G128 ? NR : 1][2][2];
+      if constexpr (G128) {
+#pragma unroll
+        for (int r = 0; r < NR; ++r)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const long long si = (long long)(min(row_of(b, h), Nout - 1) + r * Nout) * groups + s0 + l;
+            sz[r][h][0] = bf2f(__ldg(scales + si));
+            sz[r][h][1] = 1024.f + bf2f(__ldg(zeros + si));
+          }
+      }
+      float tmp[G128 ? NR : 1][NT][4];
+      if constexpr (G128) {
+#pragma unroll
+        for (int r = 0; r < NR; ++r)
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) tmp[r][nt][0] = tmp[r][nt][1] = tmp[r][nt][2] = tmp[r][nt][3] = 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < KS; ++j) {
+        uint32_t b0[NT], b1[NT];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          const uint4 xv = xs[((l * NT + nt) * CH + (j >> 1)) * 32 + lane];
+          b0[nt] = (j & 1) ? xv.z : xv.x;
+          b1[nt] = (j & 1) ? xv.w : xv.y;
+        }
+#pragma unroll
+        for (int r = 0; r < NR; ++r) {
+          const uint32_t a0 = apair<WQ>(w[r][0], j, 0), a1 = apair<WQ>(w[r][1], j, 0);
+          const uint32_t a2 = apair<WQ>(w[r][0], j, 1), a3 = apair<WQ>(w[r][1], j, 1);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            if constexpr (G128) mma16816<F16>(tmp[r][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
+            else mma16816<F16>(acc[r][nt], a0, a1, a2, a3, b0[nt], b1[nt]);
+          }
+        }
+      }
+      if constexpr (G128) {
+        // acc += s * (sum (1024 + q) x - (1024 + z) sum x) over the group
+#pragma unroll
+        for (int r = 0; r < NR; ++r)
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+              for (int cc = 0; cc < 2; ++cc) {
+                const float xsm = xsum[l * NT * 8 + nt * 8 + 2 * t + cc];
+                acc[r][nt][2 * h + cc] += sz[r][h][0] * (tmp[r][nt][2 * h + cc] - sz[r][h][1] * xsm);
+              }
+      }
+    }
+    if constexpr (WQ == FP_W_INT8) {
+      // remove the 1152 offset of the codes: acc - 1152 * sum x over the window
+#pragma unroll
+      for (int r = 0; r < NR; ++r)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) acc[r][nt][i] -= 1152.f * xsum[nt * 8 + 2 * t + (i & 1)];
+    }
+    cur += wlen;
+    if (cur < seg_end) continue;
+
+    // ---- row block b is done for this CTA
+    const long long c0 = gemv_cta_of((long long)b * S, C, total);
+    const long long c1 = gemv_cta_of((long long)(b + 1) * S - 1, C, total);
+    if (c0 == c1) {
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int row = row_of(b, i >> 1);
+          const int m = nt * 8 + 2 * t + (i & 1);
+          if (row < Nout && m < M) finish(m, row, acc[0][nt][i], acc[NR - 1][nt][i]);
+        }
+    } else {
+      // partial slot b + c: distinct for every (block, CTA) pair that meets
+      float* part = ws + (size_t)(b + c) * M * NR * ROWS;
+#pragma unroll
+      for (int r = 0; r < NR; ++r)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int lr = warp * 16 + g + 8 * (i >> 1);
+            const int m = nt * 8 + 2 * t + (i & 1);
+            if (m < M) part[((long long)m * NR + r) * ROWS + lr] = acc[r][nt][i];
+          }
+      __threadfence();
+      __syncthreads();
+      if (threadIdx.x == 0) s_last = atomicAdd(&counters[b], 1u) == (unsigned)(c1 - c0);
+      __syncthreads();
+      if (s_last) {
+        __threadfence();
+        // four rows per thread; the partial loads of several CTAs are in flight together
+        for (int idx = threadIdx.x; idx < M * (ROWS / 4); idx += blockDim.x) {
+          const int m = idx / (ROWS / 4), lr = (idx % (ROWS / 4)) * 4;
+          const size_t slot_f = (size_t)M * NR * ROWS;
+          const float* p0 = ws + (size_t)(b + c0) * slot_f + (size_t)m * NR * ROWS + lr;
+          float4 v = make_float4(0.f, 0.f, 0.f, 0.f), u = v;
+          const int cnt = (int)(c1 - c0) + 1;
+#pragma unroll 4
+          for (int cc = 0; cc < cnt; ++cc) {
+            const float4 a = __ldcg(reinterpret_cast<const float4*>(p0 + (size_t)cc * slot_f));
+            v.x += a.x, v.y += a.y, v.z += a.z, v.w += a.w;
+            if (NR == 2) {
+              const float4 e = __ldcg(reinterpret_cast<const float4*>(p0 + (size_t)cc * slot_f + ROWS));
+              u.x += e.x, u.y += e.y, u.z += e.z, u.w += e.w;
+            }
+          }
+          const float vv[4] = {v.x, v.y, v.z, v.w}, uu[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int row = b * ROWS + lr + e;
+            if (row < Nout) finish(m, row, vv[e], uu[e]);
+          }
+        }
+        if (threadIdx.x == 0) counters[b] = 0u;
+      }
+    }
+    zero_acc();
   }
-  if (threadIdx.x == 0) counters[blockIdx.x] = 0u;
+  cp_async_wait<0>();
 }
 
 // ---------------------------------------------------------------- planning
 struct GemvPlan {
-  int NT, RT, ksplit, splits, blocks;
+  int NT, ctas, S, W, blocks;
+  long long total;
   size_t smem, ws;
 };
 
 static int mma_kt(int wq) { return wq == FP_W_BF16 ? 8 : wq == FP_W_INT8 ? 16 : 32; }
 
-// Workspace = a fixed area of split-K ticket counters (zero at rest), then the
-// fp32 partials.  The ticket area has the same size for every launch, so the
+// Workspace = a fixed area of ticket counters (zero at rest), then the fp32
+// partials.  The ticket area has the same size for every launch, so the
 // partials of one launch never land on the counters of the next.
 constexpr int kTicketSlots = 4096;
 static size_t counter_bytes(int) { return (size_t)kTicketSlots * 4; }
 
-// Rows per CTA are at least 64, so N <= 64 * kTicketSlots keeps one ticket per row block.
+// One ticket per 128-row block.
 static bool mma_ok(int wq, int M, int N, int K) {
-  return M >= 1 && M <= 64 && K % (4 * mma_kt(wq)) == 0 && N <= 64 * kTicketSlots;
+  return M >= 1 && M <= 64 && K % (4 * mma_kt(wq)) == 0 && N <= kGemvWarps * 16 * kTicketSlots;
 }
 
 static int sm_count() {
@@ -555,81 +610,164 @@ static int sm_count() {
   return n;
 }
 
-// occ = resident CTAs per SM of the chosen kernel (register limited).  The
-// grid targets one full wave: blocks * splits close to SMs * occ.
-static GemvPlan plan_gemv(int wq, int epi, int M, int N, int K, int occ) {
+static int gemv_nt(int M) { return M <= 8 ? 1 : M <= 16 ? 2 : M <= 32 ? 4 : 8; }
+
+// Shared-memory limits of a kernel: per CTA (dynamic) and per SM.
+struct SmemLimits {
+  int per_cta_dyn;  // opt-in maximum minus the kernel's static shared memory
+  int per_sm;       // usable by CTAs on one SM
+  int static_bytes;
+};
+
+// occ_max = CTAs per SM the kernel's registers allow.  The plan takes the
+// most CTAs per SM whose shared memory (ring + an x window of at least a
+// third of one CTA's range, up to a whole row block) fits, and one wave of
+// CTAs.
+static GemvPlan plan_gemv(int wq, int epi, int M, int N, int K, int occ_max, const SmemLimits& lim) {
   GemvPlan p{};
   const int SUP = 4 * mma_kt(wq);
-  p.NT = M <= 8 ? 1 : M <= 16 ? 2 : M <= 32 ? 4 : 8;
-  p.RT = 1;
+  const int NT = gemv_nt(M);
   const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
   const int Nout = nr == 2 ? N / 2 : N;
-  p.blocks = (Nout + kGemvWarps * p.RT * 16 - 1) / (kGemvWarps * p.RT * 16);
-  occ = std::max(1, std::min(occ, 8));
-  // shared memory per CTA: the weight ring plus the x chunk, within 200 KiB per SM
-  const int ring = kGemvWarps * gemv_stages(nr * p.RT) * nr * p.RT * 2 * 512;
-  const int xbytes_per_k = p.NT * 8 * 2;
-  const int smem_cap = std::max(8 * 1024, std::min(96 * 1024, 200 * 1024 / occ) - ring);
-  const int kmax = std::max(SUP, (smem_cap / xbytes_per_k) / SUP * SUP);
-  // whole waves: as many splits as fit in the resident slots (at least one)
-  const int slots = sm_count() * occ;
-  const int want = std::max(1, slots / p.blocks);
-  int ks = (K + want - 1) / want;
-  ks = (ks + SUP - 1) / SUP * SUP;
-  ks = std::min(std::max(ks, SUP), kmax);
-  p.ksplit = ks;
-  p.splits = (K + ks - 1) / ks;
-  const int nsup = ks / SUP;
-  const size_t xsum_entries = wq == FP_W_BF16 ? 0 : (size_t)(wq == FP_W_INT8 ? 1 : nsup) * p.NT * 8;
-  p.smem = (size_t)nsup * p.NT * mma_kt(wq) * 64 + (xsum_entries + 3) / 4 * 16 + ring;
-  p.ws = p.splits > 1 ? counter_bytes(p.blocks) + (size_t)p.splits * M * N * 4 : 0;
+  p.NT = NT;
+  p.blocks = (Nout + kGemvWarps * 16 - 1) / (kGemvWarps * 16);
+  p.S = K / SUP;
+  p.total = (long long)p.blocks * p.S;
+  const int ring = kGemvWarps * gemv_stages(nr) * nr * 2 * 512;
+  const int per_ss = NT * SUP * 16 + (wq == FP_W_INT4_G128 ? NT * 8 * 4 : 0);  // x operands (+ int4 group sums)
+  const int fixed = wq == FP_W_INT8 ? NT * 8 * 4 : 0;                           // int8 window sums
+  const int sms = sm_count();
+  occ_max = std::max(1, std::min(occ_max, 8));
+  int best_occ = 0, best_w = 0;
+  for (int occ = occ_max; occ >= 1; --occ) {
+    const int budget = std::min(lim.per_cta_dyn, lim.per_sm / occ - 1024 - lim.static_bytes) - 16;
+    const int wmax = (budget - ring - fixed) / per_ss;
+    if (wmax < 1) continue;
+    const long long C = std::min<long long>(p.total, (long long)occ * sms);
+    const long long need = std::min<long long>((p.total + C - 1) / C, p.S);
+    if (wmax > best_w) {
+      best_w = wmax;
+      best_occ = occ;
+    }
+    if (3LL * wmax >= need) {  // at most three x windows for the longest piece of a row block
+      best_occ = occ;
+      best_w = wmax;
+      break;
+    }
+  }
+  if (best_occ == 0) return p;  // ctas == 0: no plan
+  p.ctas = (int)std::min<long long>(p.total, (long long)best_occ * sms);
+  p.W = std::min(best_w, p.S);
+  p.smem = (size_t)ring + (size_t)p.W * NT * SUP * 16 +
+           (size_t)(wq == FP_W_INT4_G128 ? p.W : (wq == FP_W_INT8 ? 1 : 0)) * NT * 8 * 4;
+  p.ws = counter_bytes(p.blocks) + (size_t)(p.blocks + p.ctas) * M * nr * kGemvWarps * 16 * 4;
   return p;
 }
 
-template <int WQ, int NT, int RT, int EPI>
-static int gemv_occupancy() {
+static int max_smem_optin() {
+  static int v = 0;
+  if (!v) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess || v <= 0)
+      v = 227 * 1024;
+  }
+  return v;
+}
+
+static int smem_per_sm() {
+  static int v = 0;
+  if (!v) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess || v <= 0)
+      v = 228 * 1024;
+  }
+  return v;
+}
+
+// CTAs per SM the kernel's registers allow, and its shared-memory limits;
+// lifts the kernel's dynamic shared memory limit to the opt-in maximum.
+template <int WQ, int NT, int EPI>
+static int gemv_occupancy(SmemLimits* lim) {
   static int occ = 0;
+  static SmemLimits l{};
   if (!occ) {
-    auto kern = gemv_mma_kernel<WQ, NT, RT, EPI>;
-    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kGemvWarps * 32, 56 * 1024) != cudaSuccess ||
-        occ <= 0)
+    auto kern = gemv_mma_kernel<WQ, NT, EPI>;
+    cudaFuncAttributes fa{};
+    int st = cudaFuncGetAttributes(&fa, kern) == cudaSuccess ? (int)fa.sharedSizeBytes : 64;
+    l.static_bytes = st;
+    l.per_cta_dyn = max_smem_optin() - st;
+    l.per_sm = smem_per_sm();
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, l.per_cta_dyn);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kGemvWarps * 32, 0) != cudaSuccess || occ <= 0)
       occ = 2;
     (void)cudaGetLastError();
   }
+  *lim = l;
   return occ;
 }
 
-template <int WQ, int NT, int RT, int EPI>
-static cudaError_t launch_mma_t(int wq, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
-                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
-                                size_t ws_bytes, cudaStream_t s) {
-  const GemvPlan p = plan_gemv(wq, epi, M, N, K, gemv_occupancy<WQ, NT, RT, EPI>());
-  // never launch with less workspace than this plan writes
-  if (p.ws > 0 && (!ws || ws_bytes < p.ws)) return cudaErrorInvalidValue;
-  auto kern = gemv_mma_kernel<WQ, NT, RT, EPI>;  // dynamic shared memory limit set by gemv_occupancy
-  if (p.smem > 200 * 1024) return cudaErrorInvalidValue;
-  unsigned* counters = (unsigned*)ws;
-  float* part = ws ? (float*)((char*)ws + counter_bytes(p.blocks)) : nullptr;
-  dim3 grid(p.blocks, p.splits);
-  return launch(kern, grid, dim3(kGemvWarps * 32), p.smem, s, x, M, N, K, codes, scales, zeros, R, y, p.ksplit,
-                p.splits, part, counters);
+template <int WQ, int NT, int EPI>
+static GemvPlan plan_t(int M, int N, int K) {
+  SmemLimits lim{};
+  const int occ = gemv_occupancy<WQ, NT, EPI>(&lim);
+  return plan_gemv(WQ, EPI, M, N, K, occ, lim);
 }
 
 template <int WQ, int EPI>
-static cudaError_t launch_mma_e(int wq, const uint16_t* x, int M, int N, int K, const void* codes,
-                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
-                                size_t ws_bytes, cudaStream_t s) {
-  const GemvPlan p = plan_gemv(wq, EPI, M, N, K, 1);  // NT and RT do not depend on occupancy
-#define FP_MMA_CASE(nt, rt) \
-  if (p.NT == nt && p.RT == rt)  \
-    return launch_mma_t<WQ, nt, rt, EPI>(wq, EPI, x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-  FP_MMA_CASE(1, 1)
-  FP_MMA_CASE(2, 1)
-  FP_MMA_CASE(4, 1)
-  FP_MMA_CASE(8, 1)
-#undef FP_MMA_CASE
-  return cudaErrorInvalidValue;
+static GemvPlan plan_e(int M, int N, int K) {
+  switch (gemv_nt(M)) {
+    case 1: return plan_t<WQ, 1, EPI>(M, N, K);
+    case 2: return plan_t<WQ, 2, EPI>(M, N, K);
+    case 4: return plan_t<WQ, 4, EPI>(M, N, K);
+    default: return plan_t<WQ, 8, EPI>(M, N, K);
+  }
+}
+
+template <int WQ>
+static GemvPlan plan_w(int epi, int M, int N, int K) {
+  switch (epi) {
+    case FP_EPI_STORE: return plan_e<WQ, FP_EPI_STORE>(M, N, K);
+    case FP_EPI_RESID: return plan_e<WQ, FP_EPI_RESID>(M, N, K);
+    case FP_EPI_SWIGLU: return plan_e<WQ, FP_EPI_SWIGLU>(M, N, K);
+    default: return plan_e<WQ, FP_EPI_F32>(M, N, K);
+  }
+}
+
+// The plan a launch of this shape uses.
+static GemvPlan plan_for(int wq, int epi, int M, int N, int K) {
+  switch (wq) {
+    case FP_W_BF16: return plan_w<FP_W_BF16>(epi, M, N, K);
+    case FP_W_INT8: return plan_w<FP_W_INT8>(epi, M, N, K);
+    default: return plan_w<FP_W_INT4_G128>(epi, M, N, K);
+  }
+}
+
+template <int WQ, int NT, int EPI>
+static cudaError_t launch_mma_t(const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
+                                const uint16_t* zeros, const uint16_t* R, void* y, void* ws, size_t ws_bytes,
+                                cudaStream_t s) {
+  const GemvPlan p = plan_t<WQ, NT, EPI>(M, N, K);
+  if (p.ctas <= 0) return cudaErrorInvalidValue;
+  // never launch with less workspace than this plan writes; partials are read as float4
+  if (!ws || ws_bytes < p.ws || ((uintptr_t)ws & 15)) return cudaErrorInvalidValue;
+  unsigned* counters = (unsigned*)ws;
+  float* part = (float*)((char*)ws + counter_bytes(p.blocks));
+  return launch(gemv_mma_kernel<WQ, NT, EPI>, dim3(p.ctas), dim3(kGemvWarps * 32), p.smem, s, x, M, N, K, codes,
+                scales, zeros, R, y, p.total, p.S, p.W, part, counters);
+}
+
+template <int WQ, int EPI>
+static cudaError_t launch_mma_e(const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
+                                const uint16_t* zeros, const uint16_t* R, void* y, void* ws, size_t ws_bytes,
+                                cudaStream_t s) {
+  switch (gemv_nt(M)) {
+    case 1: return launch_mma_t<WQ, 1, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case 2: return launch_mma_t<WQ, 2, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case 4: return launch_mma_t<WQ, 4, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    default: return launch_mma_t<WQ, 8, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+  }
 }
 
 template <int WQ>
@@ -637,10 +775,10 @@ static cudaError_t launch_mma(int epi, const uint16_t* x, int M, int N, int K, c
                               const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
                               size_t ws_bytes, cudaStream_t s) {
   switch (epi) {
-    case FP_EPI_STORE: return launch_mma_e<WQ, FP_EPI_STORE>(WQ, x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    case FP_EPI_RESID: return launch_mma_e<WQ, FP_EPI_RESID>(WQ, x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    case FP_EPI_SWIGLU: return launch_mma_e<WQ, FP_EPI_SWIGLU>(WQ, x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    default: return launch_mma_e<WQ, FP_EPI_F32>(WQ, x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case FP_EPI_STORE: return launch_mma_e<WQ, FP_EPI_STORE>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case FP_EPI_RESID: return launch_mma_e<WQ, FP_EPI_RESID>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case FP_EPI_SWIGLU: return launch_mma_e<WQ, FP_EPI_SWIGLU>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    default: return launch_mma_e<WQ, FP_EPI_F32>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
   }
 }
 
@@ -653,10 +791,10 @@ size_t linear_ws_bytes(int wquant, int M, int N, int K) {
     return w ? counter_bytes(0) + w : 0;
   }
   if (!mma_ok(wquant, M, N, K)) return 0;
-  // splits grow with occupancy, so the plan at the planner's cap (8) bounds every launch
-  size_t a = plan_gemv(wquant, FP_EPI_STORE, M, N, K, 8).ws;
-  size_t b = N % 2 == 0 ? plan_gemv(wquant, FP_EPI_SWIGLU, M, N, K, 8).ws : 0;
-  return std::max(a, b);
+  size_t w = 0;
+  for (int epi : {FP_EPI_STORE, FP_EPI_RESID, FP_EPI_F32}) w = std::max(w, plan_for(wquant, epi, M, N, K).ws);
+  if (N % 2 == 0) w = std::max(w, plan_for(wquant, FP_EPI_SWIGLU, M, N, K).ws);
+  return w;
 }
 
 size_t linear_ws_bytes_upto(int wquant, int max_m, int N, int K) {

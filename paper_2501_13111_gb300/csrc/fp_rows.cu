@@ -7,8 +7,12 @@
 // cache and its INT8 variant are a deployment configuration (Sec. 2, Sec. 3.2,
 // table "Models and configurations"); the KV cache keeps per-token decode
 // cost constant (Sec. 5.3, before Eq. 1).
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace fpk {
 
@@ -84,45 +88,83 @@ cudaError_t launch_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int 
 }
 
 // ------------------------------------------------------------------ argmax
-// One CTA per row; ties go to the lowest index.
-__global__ void argmax_kernel(const float* __restrict__ logits, int V, int32_t* __restrict__ out) {
+// A cluster of kArgmaxCTAs CTAs per row: each CTA finds the first maximum of
+// its slice, then CTA 0 of the cluster reads the slices' winners from the
+// other CTAs' shared memory (distributed shared memory) and keeps the first
+// maximum.  Ties go to the lowest index.
+constexpr int kArgmaxCTAs = 8;
+
+FP_DEV void better(float& bv, int& bi, float v, int i) {
+  if (v > bv || (v == bv && i < bi)) {
+    bv = v;
+    bi = i;
+  }
+}
+
+__global__ void __cluster_dims__(kArgmaxCTAs, 1, 1) __launch_bounds__(256)
+    argmax_kernel(const float* __restrict__ logits, int V, int32_t* __restrict__ out) {
+  __shared__ float sv[8];
+  __shared__ int si[8];
+  __shared__ float cv;
+  __shared__ int ci;
   pdl_trigger();
   pdl_wait();
-  const float* lr = logits + (long long)blockIdx.x * V;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank();
+  const int row = blockIdx.y;
+  const float* lr = logits + (long long)row * V;
+  // slices start on multiples of 4 so rows whose start is 16-byte aligned read float4s
+  const int per = ((V + kArgmaxCTAs - 1) / kArgmaxCTAs + 3) & ~3;
+  const int lo = min(V, rank * per), hi = min(V, lo + per);
   float best = -INFINITY;
   int bi = 0x7fffffff;
-  for (int i = threadIdx.x; i < V; i += blockDim.x) {
-    float v = lr[i];
-    if (v > best) { best = v; bi = i; }  // i increases per thread: strict > keeps the first
+  if ((V & 3) == 0 && ((uintptr_t)lr & 15) == 0) {
+    const float4* l4 = reinterpret_cast<const float4*>(lr);
+#pragma unroll 4
+    for (int i = (lo >> 2) + (int)threadIdx.x; i < (hi >> 2); i += blockDim.x) {
+      const float4 v = __ldg(l4 + i);
+      better(best, bi, v.x, 4 * i);
+      better(best, bi, v.y, 4 * i + 1);
+      better(best, bi, v.z, 4 * i + 2);
+      better(best, bi, v.w, 4 * i + 3);
+    }
+  } else {
+    for (int i = lo + (int)threadIdx.x; i < hi; i += blockDim.x) better(best, bi, lr[i], i);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    float ov = __shfl_xor_sync(0xffffffffu, best, o);
-    int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-    if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
+    const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    better(best, bi, ov, oi);
   }
-  __shared__ float sv[32];
-  __shared__ int si[32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) { sv[warp] = best; si[warp] = bi; }
-  __syncthreads();
-  if (warp == 0) {
-    const int nw = blockDim.x >> 5;
-    best = lane < nw ? sv[lane] : -INFINITY;
-    bi = lane < nw ? si[lane] : 0x7fffffff;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      float ov = __shfl_xor_sync(0xffffffffu, best, o);
-      int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-      if (ov > best || (ov == best && oi < bi)) { best = ov; bi = oi; }
-    }
-    if (lane == 0) out[blockIdx.x] = bi == 0x7fffffff ? 0 : bi;
+  if (lane == 0) {
+    sv[warp] = best;
+    si[warp] = bi;
   }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) better(best, bi, sv[w], si[w]);
+    cv = best;
+    ci = bi;
+  }
+  cluster.sync();  // every CTA's winner is in its shared memory
+  if (rank == 0 && threadIdx.x == 0) {
+    float b = -INFINITY;
+    int i = 0x7fffffff;
+    for (int r = 0; r < kArgmaxCTAs; ++r) {
+      const float* rv = cluster.map_shared_rank(&cv, r);
+      const int* ri = cluster.map_shared_rank(&ci, r);
+      better(b, i, *rv, *ri);
+    }
+    out[row] = i == 0x7fffffff ? 0 : i;
+  }
+  cluster.sync();  // keep the winners alive until CTA 0 has read them
 }
 
 cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  return launch(argmax_kernel, dim3(M), dim3(512), 0, s, logits, V, out);
+  return launch(argmax_kernel, dim3(kArgmaxCTAs, M), dim3(256), 0, s, logits, V, out);
 }
 
 // ------------------------------------------------------------------ RoPE + KV append

@@ -101,6 +101,23 @@ def test_linear_matches_oracle(fp, wq, m, epi):
     assert rel_err(got, ref) <= TAU[wq] / 4, (wq, m, epi, rel_err(got, ref))
 
 
+@pytest.mark.parametrize("wq", [0, 1, 2])
+@pytest.mark.parametrize("m,n,k", [(8, 272, 4096), (16, 200, 5120), (32, 136, 11008), (2, 4104, 1408)])
+def test_linear_long_k(fp, wq, m, n, k):
+    """Long K ranges per CTA (the weight pipeline wraps many times) and ragged row tiles."""
+    w = synth.weight_bf16(31 + wq, 0, 1, (n, k))
+    x = synth.uniform_bf16(32, m, (m, k), -2.0, 2.0)
+    codes, scales, zeros = _quantized_on_device(fp, wq, w)
+    _, wd = quant.quantize_weight(w, wq)
+    ref = quant.bf16_to_f32(x).astype(np.float64) @ wd.T
+    out = empty(m * n * 4)
+    ws_b = fp.fp_op_linear_workspace_bytes(wq, m, n, k)
+    ws = empty(max(ws_b, 16))
+    fp.fp_op_linear(wq, 3, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), None, ptr(out), ptr(ws), ws_b)
+    got = host(out, np.float32).reshape(m, n)
+    assert rel_err(got, ref) <= TAU[wq] / 4, (wq, m, n, k, rel_err(got, ref))
+
+
 def test_linear_residual_in_place(fp):
     m, n, k = 5, 64, 256
     w = synth.weight_bf16(3, 0, 1, (n, k))
