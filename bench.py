@@ -78,6 +78,39 @@ def kernel_bytes(a, wq, kvq, B, ctx):
     }
 
 
+# ---------------------------------------------------------------- ncu traffic
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
+# 7B-shaped decode kernels from the ncu captures summarised in profiles/
+# (microbench cases 7b-*), with the sha256 prefix of the kernel's source at
+# capture time: a changed source makes the figure stale and it is reported as
+# null.  Attention traffic is per cached token row (captured at B 8, context
+# 612) and scales with B x context.
+NCU_TRAFFIC = {
+    "attn": {"bytes": 83240704, "units": 8 * 612, "src": "fp_attention.cu", "sha": "2194d099f8f75e67"},
+    "lm_head": {"bytes": 270379776, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
+    "lin_gu": {"bytes": 94771200, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
+    "lin_qkv": {"bytes": 50478848, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
+    "lin_o": {"bytes": 16944384, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
+}
+
+
+def ncu_traffic(cls, cfg_name, B, ctx):
+    """Per-launch DRAM bytes of kernel class `cls` from the recorded capture, or None."""
+    import hashlib
+
+    t = NCU_TRAFFIC.get(cls)
+    if t is None or cfg_name != "l7b":
+        return None
+    src = os.path.join(ROOT, "paper_2501_13111_gb300", "csrc", t["src"])
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    except OSError:
+        return None
+    if sha != t["sha"]:
+        return None
+    return t["bytes"] if t["units"] is None else t["bytes"] * (B * ctx) / t["units"]
+
+
 # ---------------------------------------------------------------- clocks
 CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
            "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -328,7 +361,8 @@ def main():
                 "kernel_ms_per_step": prof["kernel_ms"],
                 "roofline": {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peak,
                              "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
-                             "bytes_per_launch": kb[dom], "launch_ms": per_launch_ms, "traffic": None},
+                             "bytes_per_launch": kb[dom], "launch_ms": per_launch_ms,
+                             "traffic": ncu_traffic(dom, args.config, B, mean_ctx)},
                 "gpu_launches": launches,
                 "clocks": clk.summary(),
                 "e2e": e2e,
