@@ -86,7 +86,7 @@ def kernel_bytes(a, wq, kvq, B, ctx):
 # null.  Attention traffic is per cached token row (captured at B 8, context
 # 612) and scales with B x context.
 NCU_TRAFFIC = {
-    "attn": {"bytes": 83240704, "units": 8 * 612, "src": "fp_attention.cu", "sha": "2194d099f8f75e67"},
+    "attn": {"bytes": 81945088, "units": 8 * 612, "src": "fp_attention.cu", "sha": "18124087fcad1249"},
     "lm_head": {"bytes": 270379776, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
     "lin_gu": {"bytes": 94771200, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
     "lin_qkv": {"bytes": 50478848, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},

@@ -10,6 +10,8 @@
 // codes enter the arithmetic exactly.
 #include <algorithm>
 
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -20,16 +22,21 @@ static constexpr float kLog2e = 1.4426950408889634f;
 // =====================================================================
 // Decode: grid (B * Hkv, splits); one CTA handles the G = H / Hkv query
 // heads of one KV head over one chunk of the context.  The chunk's K and V
-// stream through a ring of 32-token tiles in shared memory (cp.async, two
-// tiles in flight); each warp takes 8 tokens of a tile and keeps its own
-// online softmax, and the 4 warps are merged at the end.
+// stream through a ring of 64-token tiles in shared memory (cp.async, two
+// tiles in flight; rows padded so ldmatrix is conflict-free).  Each of the 4
+// warps takes 16 tokens of a tile: scores S = Q K^T and O += P V run on the
+// tensor cores (mma.sync m16n8k16, fp32 accumulation; the G query heads are
+// rows of the A operand), with an online softmax in the log2 domain on the
+// score fragments.  bf16 caches enter as they are (P in bf16); int8 codes
+// are widened exactly to fp16 in shared memory (P in fp16) and their
+// per-token scales applied in fp32 to the scores (K) and to P (V).  The 4
+// warps are merged at the end; a second kernel merges the context splits.
 // =====================================================================
-constexpr int kDecTile = 32;  // tokens per tile: two 16-token pages
-constexpr int kDecBuf = 3;    // ring depth
-constexpr int kDecOcc = 4;    // resident CTAs per SM assumed by the split geometry
+constexpr int kDecTT = 64;  // tokens per tile
+constexpr int kDecNB = 3;   // ring depth
 
 struct DecodeGeom {
-  int chunk;   // positions per split (multiple of kDecTile)
+  int chunk;   // positions per split (multiple of kDecTT)
   int splits;  // ceil(max_len / chunk)
 };
 
@@ -44,25 +51,55 @@ static int dec_sm_count() {
   return n;
 }
 
-// As many splits as fill the resident CTA slots once (whole waves), at least
-// one tile per split.  Splits never grow with n_kv_heads, so the workspace
-// sized for n_kv_heads = 1 covers every launch.
+// Resident decode CTAs per SM assumed by the split geometry (the bf16 ring
+// of 104 KB allows two).
+constexpr int kDecOcc = 2;
+
+// Split count: the candidates are the counts a whole number of tiles per
+// split produces; each is scored as (waves of resident CTAs) x (tiles per
+// split + one tile of fixed cost), and the cheapest wins (fewer splits on a
+// tie).  At most 4 splits or 2 waves' worth per (sequence, KV head) pair,
+// whichever is more (and at least the splits that keep a split within
+// kDecMaxChunkTiles tiles), so the count never grows with n_kv_heads and the
+// workspace sized for n_kv_heads = 1 covers every launch.
+constexpr int kDecMaxChunkTiles = 256;  // a split covers at most 16384 positions (bounds its page-id stage)
+
+static int dec_min_splits(int tiles) { return (tiles + kDecMaxChunkTiles - 1) / kDecMaxChunkTiles; }
+
+static int dec_max_splits(long long pairs, int tiles) {
+  const long long slots = (long long)dec_sm_count() * kDecOcc;
+  const long long s = std::max<long long>(std::min(tiles, 4), std::min<long long>(tiles, 2 * slots / std::max<long long>(1, pairs)));
+  return (int)std::max<long long>(std::max<long long>(s, 1), dec_min_splits(tiles));
+}
+
 static DecodeGeom decode_geom(int B, int n_kv_heads, int max_len) {
   const long long pairs = (long long)B * n_kv_heads;
   const long long slots = (long long)dec_sm_count() * kDecOcc;
-  const int tiles = (max_len + kDecTile - 1) / kDecTile;
-  int splits = (int)std::max<long long>(1, slots / pairs);
-  splits = std::min(splits, tiles);
-  const int per_tiles = (tiles + splits - 1) / splits;
-  DecodeGeom g;
-  g.chunk = per_tiles * kDecTile;
-  g.splits = (max_len + g.chunk - 1) / g.chunk;
-  return g;
+  const int tiles = std::max(1, (max_len + kDecTT - 1) / kDecTT);
+  const int smax = dec_max_splits(pairs, tiles);
+  DecodeGeom best{tiles * kDecTT, 1};
+  double best_t = 1e30;
+  for (int s = std::max(1, dec_min_splits(tiles)); s <= smax; ++s) {
+    const int per = (tiles + s - 1) / s;
+    const int splits = (tiles + per - 1) / per;
+    const long long ctas = pairs * splits;
+    const double t = (double)((ctas + slots - 1) / slots) * (per + 1);
+    if (t < best_t) {
+      best_t = t;
+      best.chunk = per * kDecTT;
+      best.splits = (max_len + best.chunk - 1) / best.chunk;
+    }
+  }
+  return best;
+}
+
+int attention_decode_launches(int B, int n_kv_heads, int max_len) {
+  return decode_geom(B, n_kv_heads, max_len).splits == 1 ? 1 : 2;
 }
 
 size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len) {
-  DecodeGeom g = decode_geom(B, 1, max_len);
-  size_t rows = (size_t)B * n_heads * g.splits;
+  const int tiles = std::max(1, (max_len + kDecTT - 1) / kDecTT);
+  const size_t rows = (size_t)B * n_heads * dec_max_splits(B, tiles);
   return rows * (size_t)(head_dim + 2) * sizeof(float);
 }
 
@@ -75,10 +112,70 @@ FP_DEV void dec_cp_async4(void* smem, const void* gmem) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(s), "l"(gmem) : "memory");
 }
 
+template <bool F16>
+FP_DEV void dec_mma(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  if constexpr (F16) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+  } else {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+  }
+}
+
+FP_DEV void dec_ldsm_x4(uint32_t* r, const void* p, bool trans) {
+  const uint32_t a = (uint32_t)__cvta_generic_to_shared(p);
+  if (trans)
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(a));
+  else
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(a));
+}
+
+// Two fp32 values as an MMA operand word: bf16 or fp16 pair.
+template <bool F16>
+FP_DEV uint32_t dec_pack(float a, float b) {
+  if constexpr (F16) {
+    const __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&h);
+  } else {
+    return pack_bf2(a, b);
+  }
+}
+
+// int8 codes (4 per word) -> two fp16 pairs, exactly: fp16(1024 + (q + 128)) - 1152.
+FP_DEV uint2 dec_i8_to_f16x4(uint32_t w) {
+  const uint32_t x = w ^ 0x80808080u;
+  const uint32_t lo = __byte_perm(x, 0x64646464u, 0x5140), hi = __byte_perm(x, 0x64646464u, 0x5342);
+  const __half2 off = __float2half2_rn(1152.f);
+  const __half2 a = __hsub2(*reinterpret_cast<const __half2*>(&lo), off);
+  const __half2 b = __hsub2(*reinterpret_cast<const __half2*>(&hi), off);
+  return make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&b));
+}
+
 template <int HD, int KVQ>
 constexpr size_t dec_smem_bytes() {
-  return (size_t)kDecBuf * kDecTile * HD * (KVQ == FP_KV_BF16 ? 2 : 1) * 2 +
-         (KVQ == FP_KV_INT8 ? (size_t)kDecBuf * kDecTile * 2 * sizeof(float) : 0);
+  constexpr size_t ld = HD + 8;  // padded 16-bit row (elements)
+  if (KVQ == FP_KV_BF16) return (size_t)kDecNB * kDecTT * ld * 2 * 2;
+  // int8: ring of code rows (HD + 16 bytes), per-token scales, one fp16 tile of K and V
+  return (size_t)kDecNB * kDecTT * (HD + 16) * 2 + (size_t)kDecNB * kDecTT * 2 * sizeof(float) +
+         (size_t)kDecTT * ld * 2 * 2;
+}
+
+// The ring, which also holds the 4-warp merge buffer after the loop; the
+// chunk's page ids follow it.
+template <int HD, int KVQ, int G>
+constexpr size_t dec_stage_bytes() {
+  return std::max(dec_smem_bytes<HD, KVQ>(), (size_t)4 * G * (HD + 2) * sizeof(float));
 }
 
 // Workspace layout for (b, h, split): o [HD] fp32 (un-normalised, relative to
@@ -87,16 +184,22 @@ template <int HD, int KVQ, int G>
 __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __restrict__ q, int q_stride, int H,
                                                           fp_kv_view kv, const int32_t* __restrict__ len,
                                                           int len_add, int max_len, int chunk, int splits,
-                                                          float* __restrict__ ws, int32_t* err) {
-  constexpr int TT = kDecTile, NBUF = kDecBuf;
-  constexpr int ELT = KVQ == FP_KV_BF16 ? 2 : 1, ROWB = HD * ELT, TILEB = TT * ROWB, CPR = ROWB / 16;
-  constexpr int DPL = HD / 32;                   // dims per lane
-  constexpr int TG = G >= 4 ? 2 : (G == 2 ? 4 : 8);  // tokens per softmax update
+                                                          float* __restrict__ ws, uint16_t* __restrict__ out,
+                                                          int32_t* err) {
+  constexpr int TT = kDecTT, NB = kDecNB, LD = HD + 8;
+  constexpr bool I8 = KVQ == FP_KV_INT8;
+  constexpr int RAWB = I8 ? HD + 16 : LD * 2;  // bytes per staged row
+  constexpr int CPR = (I8 ? HD : HD * 2) / 16;  // 16-byte chunks per row
+  constexpr int NT = HD / 8;                    // n8 tiles of the output
+  static_assert(G <= 8, "query heads per KV head are rows 0..7 of the MMA tile");
+  static_assert(TT == 4 * 16, "each of the 4 warps takes 16 tokens of a tile");
   extern __shared__ __align__(16) uint8_t smem[];
-  uint8_t* sK = smem;                  // [NBUF][TT][ROWB]
-  uint8_t* sV = sK + NBUF * TILEB;     // [NBUF][TT][ROWB]
-  float* sKs = reinterpret_cast<float*>(sV + NBUF * TILEB);  // int8: [NBUF][TT]
-  float* sVs = sKs + NBUF * TT;
+  uint8_t* sK = smem;                                          // [NB][TT][RAWB]
+  uint8_t* sV = sK + NB * TT * RAWB;                           // [NB][TT][RAWB]
+  float* sKs = reinterpret_cast<float*>(sV + NB * TT * RAWB);  // int8: [NB][TT]
+  float* sVs = sKs + NB * TT;
+  uint16_t* cK = reinterpret_cast<uint16_t*>(sVs + NB * TT);  // int8: fp16 [TT][LD]
+  uint16_t* cV = cK + TT * LD;
   pdl_trigger();
   pdl_wait();
   const int Hkv = kv.n_kv_heads;
@@ -108,177 +211,209 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __rest
     T = max_len;
   }
   const int t0 = split * chunk;
-  if (t0 >= T) return;
+  if (t0 >= T) {
+    if (splits == 1)  // empty context: zero output
+      for (int i = threadIdx.x; i < G * HD; i += 128) out[((long long)b * H + kvh * G) * HD + i] = 0;
+    return;
+  }
   const int t1 = min(T, t0 + chunk);
   const int ntile = (t1 - t0 + TT - 1) / TT;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
+  // ---- the page ids of positions t0 .. t1-1, staged once (past the table: -1)
+  int* spt = reinterpret_cast<int*>(smem + dec_stage_bytes<HD, KVQ, G>());
+  {
+    const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
+    const int lp0 = t0 / kv.page_size, n = (t1 - 1) / kv.page_size - lp0 + 1;
+    for (int i = tid; i < n; i += 128) spt[i] = lp0 + i < kv.pages_per_seq ? pt[lp0 + i] : -1;
+    __syncthreads();
+  }
+  const int lp0 = t0 / kv.page_size;
 
-  // ---- issue one tile of K, V (and their int8 scales) into ring slot tile % NBUF
+  // ---- one tile of K, V (and their int8 scales) into ring slot tile % NB.
+  // Rows of tokens at or past t1 (or with a bad page) are zero-filled, so
+  // their (masked) scores and zero probabilities meet finite values.  Each
+  // thread copies the same 16-byte column of rows jb, jb + RPP, ...; page
+  // arithmetic is shifts and masks when the page size is a power of two.
+  constexpr int RPP = 128 / CPR, PASSES = TT / RPP;
+  static_assert(128 % CPR == 0 && TT % RPP == 0, "row split of the tile copy");
+  const int part = tid % CPR, jb = tid / CPR;
+  const int P = kv.page_size;
+  const bool pow2 = (P & (P - 1)) == 0;
+  const int lgP = __ffs(P) - 1;
+  auto page_of = [&](int t) { return pow2 ? t >> lgP : t / P; };
+  auto slot_in_page = [&](int t) { return pow2 ? t & (P - 1) : t % P; };
   auto issue = [&](int tile) {
     const int tt0 = t0 + tile * TT;
-    uint8_t* dK = sK + (tile % NBUF) * TILEB;
-    uint8_t* dV = sV + (tile % NBUF) * TILEB;
-    for (int c = tid; c < TT * CPR; c += 128) {
-      const int j = c / CPR, part = c % CPR, t = tt0 + j;
-      const int lp = t / kv.page_size;
-      if (lp >= kv.pages_per_seq) continue;  // past the sequence's table: masked below
-      const int page = pt[lp];
-      uint8_t* dk = dK + j * ROWB + part * 16;
-      uint8_t* dv = dV + j * ROWB + part * 16;
+    uint8_t* dK = sK + (tile % NB) * TT * RAWB + part * 16;
+    uint8_t* dV = sV + (tile % NB) * TT * RAWB + part * 16;
+#pragma unroll
+    for (int k = 0; k < PASSES; ++k) {
+      const int j = jb + k * RPP, t = tt0 + j;
+      const int page = t < t1 ? spt[page_of(t) - lp0] : -1;
       if (page < 0 || page >= kv.n_pages) {
         if (err && t < t1) atomicExch(err, 1);
+        *reinterpret_cast<uint4*>(dK + j * RAWB) = make_uint4(0, 0, 0, 0);
+        *reinterpret_cast<uint4*>(dV + j * RAWB) = make_uint4(0, 0, 0, 0);
         continue;
       }
-      const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
-      dec_cp_async16(dk, (const uint8_t*)kv.k_pool + rowi * ROWB + part * 16);
-      dec_cp_async16(dv, (const uint8_t*)kv.v_pool + rowi * ROWB + part * 16);
+      const long long off = (((long long)page * Hkv + kvh) * P + slot_in_page(t)) * (I8 ? HD : HD * 2) + part * 16;
+      dec_cp_async16(dK + j * RAWB, (const uint8_t*)kv.k_pool + off);
+      dec_cp_async16(dV + j * RAWB, (const uint8_t*)kv.v_pool + off);
     }
-    if constexpr (KVQ == FP_KV_INT8) {
-      for (int j = tid; j < TT; j += 128) {
-        const int t = tt0 + j, lp = t / kv.page_size;
-        if (lp >= kv.pages_per_seq) continue;
-        const int page = pt[lp];
-        if (page < 0 || page >= kv.n_pages) continue;
-        const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
-        dec_cp_async4(sKs + (tile % NBUF) * TT + j, kv.k_scale + rowi);
-        dec_cp_async4(sVs + (tile % NBUF) * TT + j, kv.v_scale + rowi);
+    if constexpr (I8) {
+      if (tid < TT) {
+        const int j = tid, t = tt0 + j;
+        const int page = t < t1 ? spt[page_of(t) - lp0] : -1;
+        float* ks = sKs + (tile % NB) * TT + j;
+        float* vs = sVs + (tile % NB) * TT + j;
+        if (page < 0 || page >= kv.n_pages) {
+          *ks = 0.f;
+          *vs = 0.f;
+        } else {
+          const long long rowi = ((long long)page * Hkv + kvh) * P + slot_in_page(t);
+          dec_cp_async4(ks, kv.k_scale + rowi);
+          dec_cp_async4(vs, kv.v_scale + rowi);
+        }
       }
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
   };
 #pragma unroll
-  for (int i = 0; i < NBUF - 1; ++i) {
+  for (int i = 0; i < NB - 1; ++i) {
     if (i < ntile) issue(i);
     else asm volatile("cp.async.commit_group;" ::: "memory");
   }
 
-  // q of the G heads, this lane's dims, pre-scaled by log2(e) / sqrt(hd)
-  const float qscale = kLog2e * rsqrtf((float)HD);
-  float qr[G][DPL];
+  // q of the G heads as the A operand: row g8 = head kvh G + g8 (rows >= G and
+  // g8 + 8 are zero); bf16 as stored, or widened to fp16 for the int8 cache
+  const int g8 = lane >> 2, t4 = lane & 3;
+  uint32_t qa[HD / 16][4];
+  {
+    const uint16_t* qh = q + (long long)b * q_stride + (long long)(kvh * G + g8) * HD;
 #pragma unroll
-  for (int g = 0; g < G; ++g)
-#pragma unroll
-    for (int d = 0; d < DPL; ++d)
-      qr[g][d] = bf2f(q[(long long)b * q_stride + (long long)(kvh * G + g) * HD + lane * DPL + d]) * qscale;
-  float m[G], l[G], acc[G][DPL];
-#pragma unroll
-  for (int g = 0; g < G; ++g) {
-    m[g] = -INFINITY;
-    l[g] = 0.f;
-#pragma unroll
-    for (int d = 0; d < DPL; ++d) acc[g][d] = 0.f;
+    for (int ks = 0; ks < HD / 16; ++ks) {
+      uint32_t lo = 0, hi = 0;
+      if (g8 < G) {
+        const uint16_t* qp = qh + ks * 16 + 2 * t4;  // q_stride may be odd: 16-bit loads
+        lo = (uint32_t)qp[0] | ((uint32_t)qp[1] << 16);
+        hi = (uint32_t)qp[8] | ((uint32_t)qp[9] << 16);
+        if constexpr (I8) {
+          const float2 a = bf2x2f(lo), c = bf2x2f(hi);
+          lo = dec_pack<true>(a.x, a.y);
+          hi = dec_pack<true>(c.x, c.y);
+        }
+      }
+      qa[ks][0] = lo;
+      qa[ks][1] = 0u;
+      qa[ks][2] = hi;
+      qa[ks][3] = 0u;
+    }
   }
+  const float scale = kLog2e * rsqrtf((float)HD);
+  float o[NT][4];
+#pragma unroll
+  for (int i = 0; i < NT; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m = -INFINITY, l = 0.f;  // row g8 (this lane's partial l)
+  const int j0 = warp * 16;
 
   for (int tile = 0; tile < ntile; ++tile) {
-    asm volatile("cp.async.wait_group %0;" ::"n"(NBUF - 2) : "memory");
+    asm volatile("cp.async.wait_group %0;" ::"n"(NB - 2) : "memory");
     __syncthreads();  // tile landed for every thread; the slot refilled below is free
-    if (tile + NBUF - 1 < ntile) issue(tile + NBUF - 1);
+    if (tile + NB - 1 < ntile) issue(tile + NB - 1);
     else asm volatile("cp.async.commit_group;" ::: "memory");
-    const int slot = tile % NBUF;
-    const uint8_t* tK = sK + slot * TILEB;
-    const uint8_t* tV = sV + slot * TILEB;
+    const int slot = tile % NB;
+    const uint16_t* tK;
+    const uint16_t* tV;
+    if constexpr (I8) {
+      // widen the tile's codes to fp16 (exact); scales stay per token
+      const uint8_t* rk = sK + slot * TT * RAWB;
+      const uint8_t* rv = sV + slot * TT * RAWB;
+      for (int c = tid; c < TT * HD / 4; c += 128) {
+        const int row = c / (HD / 4), col = (c % (HD / 4)) * 4;
+        *reinterpret_cast<uint2*>(cK + row * LD + col) = dec_i8_to_f16x4(*reinterpret_cast<const uint32_t*>(rk + row * RAWB + col));
+        *reinterpret_cast<uint2*>(cV + row * LD + col) = dec_i8_to_f16x4(*reinterpret_cast<const uint32_t*>(rv + row * RAWB + col));
+      }
+      __syncthreads();
+      tK = cK;
+      tV = cV;
+    } else {
+      tK = reinterpret_cast<const uint16_t*>(sK + slot * TT * RAWB);
+      tV = reinterpret_cast<const uint16_t*>(sV + slot * TT * RAWB);
+    }
     const int tt0 = t0 + tile * TT;
+    if (tt0 + j0 < t1) {  // this warp has valid tokens in the tile (warp-uniform)
+      // ---- S = Q K^T over this warp's 16 tokens: two n8 tiles
+      float s[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
-    for (int grp = 0; grp < 8 / TG; ++grp) {
-      float sc[TG][G];
-#pragma unroll
-      for (int i = 0; i < TG; ++i) {
-        const int j = warp * 8 + grp * TG + i;
-        if (tt0 + j < t1) {  // warp-uniform
-          float kf[DPL];
-          if constexpr (KVQ == FP_KV_BF16) {
-            if constexpr (DPL == 4) {
-              const uint2 raw = *reinterpret_cast<const uint2*>(tK + j * ROWB + lane * 8);
-              const float2 a = bf2x2f(raw.x), c = bf2x2f(raw.y);
-              kf[0] = a.x; kf[1] = a.y; kf[2] = c.x; kf[3] = c.y;
-            } else {
-              const float2 a = bf2x2f(*reinterpret_cast<const uint32_t*>(tK + j * ROWB + lane * 4));
-              kf[0] = a.x; kf[1] = a.y;
-            }
-          } else {
-            uint32_t raw;
-            if constexpr (DPL == 4) raw = *reinterpret_cast<const uint32_t*>(tK + j * ROWB + lane * 4);
-            else raw = *reinterpret_cast<const uint16_t*>(tK + j * ROWB + lane * 2);
-#pragma unroll
-            for (int d = 0; d < DPL; ++d) kf[d] = (float)(int8_t)((raw >> (8 * d)) & 0xFF);
-          }
-          const float ks = KVQ == FP_KV_INT8 ? sKs[slot * TT + j] : 1.f;
-#pragma unroll
-          for (int g = 0; g < G; ++g) {
-            float a = 0.f;
-#pragma unroll
-            for (int d = 0; d < DPL; ++d) a += qr[g][d] * kf[d];
-            sc[i][g] = warp_sum(a) * ks;
-          }
-        } else {
-#pragma unroll
-          for (int g = 0; g < G; ++g) sc[i][g] = -INFINITY;
-        }
+      for (int ks = 0; ks < HD / 16; ++ks) {
+        uint32_t r[4];  // (tokens 0-7 | 8-15) x (dims lo | hi) of this k-step
+        dec_ldsm_x4(r, tK + (j0 + ((lane >> 4) << 3) + (lane & 7)) * LD + ks * 16 + ((lane >> 3) & 1) * 8, false);
+        dec_mma<I8>(s[0], qa[ks], r[0], r[1]);
+        dec_mma<I8>(s[1], qa[ks], r[2], r[3]);
       }
-      // online softmax over these TG tokens
-      float p[TG][G];
+      // ---- online softmax on row g8 (columns 2 t4, 2 t4 + 1 of each n8 tile)
+      float sc[4];
 #pragma unroll
-      for (int g = 0; g < G; ++g) {
-        float mx = m[g];
+      for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
-        for (int i = 0; i < TG; ++i) mx = fmaxf(mx, sc[i][g]);
-        const float ref = mx == -INFINITY ? 0.f : mx;
-        const float corr = exp2f(m[g] - ref);
-        float ps = 0.f;
-#pragma unroll
-        for (int i = 0; i < TG; ++i) {
-          p[i][g] = exp2f(sc[i][g] - ref);
-          ps += p[i][g];
+        for (int c = 0; c < 2; ++c) {
+          const int tok = j0 + nt * 8 + 2 * t4 + c;
+          float v = s[nt][c] * scale;
+          if constexpr (I8) v *= sKs[slot * TT + tok];
+          sc[nt * 2 + c] = tt0 + tok < t1 ? v : -INFINITY;
         }
-        l[g] = l[g] * corr + ps;
-        m[g] = mx;
+      float mx = fmaxf(fmaxf(sc[0], sc[1]), fmaxf(sc[2], sc[3]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float mnew = fmaxf(m, mx);
+      const float ref = mnew == -INFINITY ? 0.f : mnew;
+      const float corr = exp2f(m - ref);
+      float p[4], ps = 0.f;
 #pragma unroll
-        for (int d = 0; d < DPL; ++d) acc[g][d] *= corr;
+      for (int i = 0; i < 4; ++i) {
+        p[i] = exp2f(sc[i] - ref);
+        ps += p[i];
       }
+      l = l * corr + ps;
+      m = mnew;
 #pragma unroll
-      for (int i = 0; i < TG; ++i) {
-        const int j = warp * 8 + grp * TG + i;
-        if (tt0 + j < t1) {
-          float vf[DPL];
-          if constexpr (KVQ == FP_KV_BF16) {
-            if constexpr (DPL == 4) {
-              const uint2 raw = *reinterpret_cast<const uint2*>(tV + j * ROWB + lane * 8);
-              const float2 a = bf2x2f(raw.x), c = bf2x2f(raw.y);
-              vf[0] = a.x; vf[1] = a.y; vf[2] = c.x; vf[3] = c.y;
-            } else {
-              const float2 a = bf2x2f(*reinterpret_cast<const uint32_t*>(tV + j * ROWB + lane * 4));
-              vf[0] = a.x; vf[1] = a.y;
-            }
-          } else {
-            uint32_t raw;
-            if constexpr (DPL == 4) raw = *reinterpret_cast<const uint32_t*>(tV + j * ROWB + lane * 4);
-            else raw = *reinterpret_cast<const uint16_t*>(tV + j * ROWB + lane * 2);
-            const float vs = sVs[slot * TT + j];
+      for (int i = 0; i < NT; ++i) {
+        o[i][0] *= corr;
+        o[i][1] *= corr;
+      }
+      if constexpr (I8) {
 #pragma unroll
-            for (int d = 0; d < DPL; ++d) vf[d] = (float)(int8_t)((raw >> (8 * d)) & 0xFF) * vs;
-          }
+        for (int i = 0; i < 4; ++i) p[i] *= sVs[slot * TT + j0 + (i >> 1) * 8 + 2 * t4 + (i & 1)];
+      }
+      // P as the A operand over k = this warp's 16 tokens (row g8 only)
+      const uint32_t pa[4] = {dec_pack<I8>(p[0], p[1]), 0u, dec_pack<I8>(p[2], p[3]), 0u};
+      // ---- O += P V: V^T fragments by transposing ldmatrix, two n8 tiles per step
 #pragma unroll
-          for (int g = 0; g < G; ++g)
-#pragma unroll
-            for (int d = 0; d < DPL; ++d) acc[g][d] += p[i][g] * vf[d];
-        }
+      for (int dn = 0; dn < HD / 16; ++dn) {
+        uint32_t r[4];  // (tokens 0-7 | 8-15) x (dims +0..7 | +8..15)
+        dec_ldsm_x4(r, tV + (j0 + ((lane >> 3) & 1) * 8 + (lane & 7)) * LD + dn * 16 + (lane >> 4) * 8, true);
+        dec_mma<I8>(o[2 * dn], pa, r[0], r[1]);
+        dec_mma<I8>(o[2 * dn + 1], pa, r[2], r[3]);
       }
     }
   }
   asm volatile("cp.async.wait_group 0;" ::: "memory");
+  l += __shfl_xor_sync(0xffffffffu, l, 1);
+  l += __shfl_xor_sync(0xffffffffu, l, 2);
   __syncthreads();  // the ring is reused for the merge below
 
-  // ---- merge the 4 warps: per head, o = sum_w acc_w 2^(m_w - M), l = sum_w l_w 2^(m_w - M)
+  // ---- merge the 4 warps: per head, o = sum_w o_w 2^(m_w - M), l = sum_w l_w 2^(m_w - M)
   float* red = reinterpret_cast<float*>(smem);  // [4][G][HD + 2]
+  if (g8 < G) {
+    float* r = red + (warp * G + g8) * (HD + 2);
 #pragma unroll
-  for (int g = 0; g < G; ++g) {
-    float* r = red + (warp * G + g) * (HD + 2);
-#pragma unroll
-    for (int d = 0; d < DPL; ++d) r[lane * DPL + d] = acc[g][d];
-    if (lane == 0) {
-      r[HD] = m[g];
-      r[HD + 1] = l[g];
+    for (int i = 0; i < NT; ++i) {
+      r[i * 8 + 2 * t4] = o[i][0];
+      r[i * 8 + 2 * t4 + 1] = o[i][1];
+    }
+    if (t4 == 0) {
+      r[HD] = m;
+      r[HD + 1] = l;
     }
   }
   __syncthreads();
@@ -287,17 +422,21 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __rest
     float M = -INFINITY;
 #pragma unroll
     for (int w = 0; w < 4; ++w) M = fmaxf(M, red[(w * G + g) * (HD + 2) + HD]);
-    float o = 0.f, L = 0.f;
+    float ov = 0.f, L = 0.f;
 #pragma unroll
     for (int w = 0; w < 4; ++w) {
       const float* r = red + (w * G + g) * (HD + 2);
       const float f = r[HD] == -INFINITY ? 0.f : exp2f(r[HD] - M);
-      o += r[e] * f;
+      ov += r[e] * f;
       L += r[HD + 1] * f;
+    }
+    if (splits == 1) {  // the whole context: normalise here, no combine pass
+      out[((long long)b * H + kvh * G + g) * HD + e] = f2bf(ov / L);
+      continue;
     }
     const long long row = ((long long)b * H + kvh * G + g) * splits + split;
     float* w = ws + row * (HD + 2);
-    w[e] = o;
+    w[e] = ov;
     if (e == 0) {
       w[HD] = M;
       w[HD + 1] = L;
@@ -333,13 +472,13 @@ static cudaError_t launch_decode_t(const uint16_t* q, int q_stride, int B, int H
                                    const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
                                    uint16_t* out, int32_t* err, cudaStream_t s, cudaError_t* second) {
   // the ring also holds the 4-warp merge buffer after the loop
-  const size_t smem = std::max(dec_smem_bytes<HD, KVQ>(), (size_t)4 * G * (HD + 2) * sizeof(float));
+  const size_t smem = dec_stage_bytes<HD, KVQ, G>() + ((size_t)g.chunk / kv.page_size + 2) * sizeof(int);
   auto kern = attn_decode_kernel<HD, KVQ, G>;
   if (smem > 48 * 1024) FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   dim3 grid(B * kv.n_kv_heads, g.splits);
   cudaError_t e = launch(kern, grid, dim3(128), smem, s, q, q_stride, H, kv, len, len_add, max_len, g.chunk,
-                         g.splits, ws, err);
-  if (e != cudaSuccess) return e;
+                         g.splits, ws, out, err);
+  if (e != cudaSuccess || g.splits == 1) return e;
   e = launch(attn_combine_kernel<HD>, dim3(B * H), dim3(HD), 0, s, H, len, len_add, max_len, g.chunk, g.splits,
              (const float*)ws, out);
   if (second) *second = e;

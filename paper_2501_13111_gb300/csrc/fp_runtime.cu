@@ -300,8 +300,8 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
       cudaError_t e = launch_attention_decode(h->qkv, h->n_qkv, B, a.n_heads, kv, h->pos, 1, h->T, h->att,
                                               h->attn_ws, h->err, s, &e2);
       if (e != cudaSuccess) return h->cuda_fail(e, "attention decode");
-      // the split kernel and the combine kernel are timed together
-      h->launches += 2;
+      // the split kernel and the combine kernel (when there is one) are timed together
+      h->launches += attention_decode_launches(B, a.n_kv_heads, h->T);
       h->tr.after(FP_K_ATTN);
     } else {
       LTRY(launch_attention_prefill(h->qkv, h->n_qkv, B, S, a.n_heads, kv, h->att, h->err, s), FP_K_ATTN);

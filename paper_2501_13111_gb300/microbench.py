@@ -161,6 +161,7 @@ RUNNERS = {"linear": case_linear, "attention": case_attention, "argmax": case_ar
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--only", default=None, help="run one case (single copy, for a profiler capture)")
+    ap.add_argument("--cases", default=None, help="comma-separated cases to run (L2-defeating copies)")
     ap.add_argument("--iters", type=int, default=10)
     ap.add_argument("--json", default=None, help="write the results here")
     ap.add_argument("--list", action="store_true")
@@ -170,7 +171,7 @@ def main(argv=None):
             print(k, kind, a)
         return
     torch.cuda.set_device(0)
-    names = [args.only] if args.only else list(CASES)
+    names = [args.only] if args.only else (args.cases.split(",") if args.cases else list(CASES))
     res = {}
     for name in names:
         kind, a = CASES[name]

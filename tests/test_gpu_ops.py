@@ -212,8 +212,8 @@ class Cache:
 
 
 @pytest.mark.parametrize("kvq", [0, 1])
-@pytest.mark.parametrize("hd,H,Hkv", [(64, 8, 8), (128, 8, 1), (128, 64, 8), (128, 4, 2)])
-@pytest.mark.parametrize("lens", [[1], [17, 300, 16], [1037, 5]])
+@pytest.mark.parametrize("hd,H,Hkv", [(64, 8, 8), (128, 8, 1), (128, 64, 8), (128, 4, 2), (128, 16, 4)])
+@pytest.mark.parametrize("lens", [[1], [17, 300, 16], [1037, 5], [4000, 63, 2500]])
 def test_attention_decode(fp, kvq, hd, H, Hkv, lens):
     B, T = len(lens), max(lens) + 3
     c = Cache(fp, kvq, B, T, Hkv, hd, seed=hd + H + kvq)

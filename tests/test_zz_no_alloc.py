@@ -56,7 +56,7 @@ def test_noalloc_rejects_requests_beyond_its_scratch():
     """Checked on the host before any CUDA call: runs without a GPU."""
     import paper_2501_13111_gb300 as fp
 
-    B, H, hd, max_len = 1, 128, 128, 19200
+    B, H, hd, max_len = 1, 128, 128, 40000
     assert fp.fp_op_attention_decode_workspace_bytes(B, H, hd, max_len) > fp.FP_NOALLOC_SCRATCH_BYTES
     kv = fp.fp_kv_view(0, 16, hd, 16, (max_len + 15) // 16, B * ((max_len + 15) // 16), 1, 1, None, None, 1)
     code = fp._lib.fp_op_attention_decode_noalloc(1, H * hd, B, H, ctypes.byref(kv), 1, max_len, 1, None, None)
