@@ -138,7 +138,7 @@ def tensor_shape(arch: Arch, layer: int, tensor: int):
             (d,), (f, d), (f, d), (d, f)][tensor]
 
 
-def build_weights(arch: Arch, wquant: int, get_bf16):
+def build_weights(arch: Arch, wquant: int, get_bf16, map_fn=map):
     """Quantise bf16 weights the way the configuration says.
 
     get_bf16(layer, tensor, shape) -> bf16 bit patterns.  Linear layers of
@@ -146,11 +146,14 @@ def build_weights(arch: Arch, wquant: int, get_bf16):
     Wqkv = [Wq; Wk; Wv] and Wgu = [Wgate; Wup] (row-wise quantisers, so
     fusing changes no code).  Embedding, norm gains and the LM head stay
     bf16.  Returns (fp64 weights for the forward pass, quantised payloads).
+    ``map_fn`` applies the quantiser to the matrices (a thread pool's map
+    spreads the large ones over cores; the result does not depend on it).
     """
     w, payload = {}, {}
     f64 = lambda b: quant.bf16_to_f32(b).astype(np.float64)
     for t, name in enumerate(GLOBAL_TENSORS):
         w[name] = f64(get_bf16(-1, t, tensor_shape(arch, -1, t)))
+    jobs = []
     for l in range(arch.n_layers):
         raw = {name: get_bf16(l, t, tensor_shape(arch, l, t)) for t, name in enumerate(LAYER_TENSORS)}
         w[(l, "attn_norm")] = f64(raw["attn_norm"])
@@ -159,8 +162,9 @@ def build_weights(arch: Arch, wquant: int, get_bf16):
                 "wo": raw["wo"],
                 "wgu": np.concatenate([raw["wgate"], raw["wup"]]),
                 "wdown": raw["wdown"]}
-        for name, bits in mats.items():
-            payload[(l, name)], w[(l, name)] = quant.quantize_weight(bits, wquant)
+        jobs += [((l, name), bits) for name, bits in mats.items()]
+    for (key, _), res in zip(jobs, map_fn(lambda j: quant.quantize_weight(j[1], wquant), jobs)):
+        payload[key], w[key] = res
     return w, payload
 
 

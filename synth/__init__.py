@@ -23,6 +23,8 @@ in ``paper_2501_13111_gb300/csrc/fp_quant.cu`` and ``common.cuh``):
 """
 from __future__ import annotations
 
+import os
+
 import numpy as np
 
 GAMMA = 0x9E3779B97F4A7C15
@@ -95,11 +97,22 @@ def normal_bf16(seed: int, stream: int, start: int, count: int) -> np.ndarray:
     """bf16 bit patterns of approximately N(0, 0.02) weights (see module doc)."""
     out = np.empty(count, dtype=np.uint16)
     step = 1 << 20  # chunks that stay in cache
-    for lo in range(0, count, step):
+
+    def chunk(lo):
         n = min(step, count - lo)
         s = _irwin_hall_sum(draws(seed, stream, start + lo, n))
         v = (s - IRWIN_HALL_MEAN).astype(np.float64) * WEIGHT_SCALE_002
         out[lo:lo + n] = f32_to_bf16_bits(v.astype(np.float32))
+
+    starts = range(0, count, step)
+    if count >= 8 * step:  # counter-based draws: chunks are independent, numpy releases the GIL
+        from concurrent.futures import ThreadPoolExecutor
+
+        with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
+            list(ex.map(chunk, starts))
+    else:
+        for lo in starts:
+            chunk(lo)
     return out
 
 
