@@ -235,6 +235,37 @@ def config_json(args, cfg):
             "l2": "inputs larger than L2 (every decode step streams all block weights and the LM head)"}
 
 
+# ---------------------------------------------------------------- sweep
+SWEEP_ARCH = (1, 8192, 64, 8, 128, 28672, 32000)  # the 70B-shaped block with embedding and LM head
+
+
+def run_sweep(args):
+    """The configuration sweep: weights x KV x batch x context on the 70B-shaped
+    block, fp_profile (device events) per point; one JSON line per point."""
+    import torch
+
+    import paper_2501_13111_gb300 as fp
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    a = arch_dict(SWEEP_ARCH)
+    N = 100
+    for wq in (0, 1, 2):
+        for kvq in (0, 1):
+            for B in (1, 8, 32, 64):
+                for ctx in (128, 512, 2048, 4096):
+                    h = fp.fp_create(a, wq, kvq, B, ctx + N + 1, seed=0)
+                    try:
+                        r = fp.fp_profile(h, ctx, N, warmup=1, iters=1).as_dict()
+                    finally:
+                        fp.fp_destroy(h)
+                    print(json.dumps({"weights": WQ_NAME[wq], "kv_cache": KV_NAME[kvq], "batch": B, "context": ctx,
+                                      "decode_tokens": N, "ttft_ms": r["ttft_ms"], "tpot_ms": r["tpot_ms"],
+                                      "decode_tokens_per_s": r["decode_tokens_per_s"],
+                                      "peak_hbm_bytes": r["peak_hbm_bytes"],
+                                      "decode_bytes_per_step": r["decode_bytes_per_step"]}), flush=True)
+    return 0
+
+
 # ---------------------------------------------------------------- our arm
 def main():
     ap = argparse.ArgumentParser()
@@ -245,7 +276,10 @@ def main():
     ap.add_argument("--config", default="l7b", choices=list(CONFIGS))
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass (profiling runs)")
+    ap.add_argument("--sweep", action="store_true", help="profile the 96-point configuration sweep instead")
     args = ap.parse_args()
+    if args.sweep:
+        return run_sweep(args)
     cfg = CONFIGS[args.config]
     if args.impl == "reference":
         return run_reference(args, cfg)

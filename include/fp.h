@@ -199,7 +199,9 @@ int fp_profile(fp_handle* h, int prompt_len, int n_decode, int warmup, int iters
                const int32_t* host_prompt, fp_profile_result* out);
 
 /* Reads for tests (synchronous).  Returns bytes written, or the size needed
- * when host_dst is NULL, or an FP_ERR_* code.  `mat` picks a fused matrix:
+ * when host_dst is NULL, or an FP_ERR_* code.  A host buffer smaller than the
+ * tensor receives its leading `bytes` bytes (e.g. the first rows of
+ * FP_G_HIDDEN, which are sequence 0's).  `mat` picks a fused matrix:
  * FP_M_QKV = [Wq; Wk; Wv], FP_M_O, FP_M_GU = [Wgate; Wup], FP_M_DOWN. */
 enum { FP_M_QKV = 0, FP_M_O = 1, FP_M_GU = 2, FP_M_DOWN = 3 };
 enum {

@@ -227,12 +227,14 @@ def fp_profile(h, prompt_len, n_decode, warmup=1, iters=3, prompt=None):
     return res
 
 
-def fp_get_tensor(h, what, layer=0, mat=0, dtype=None):
-    """With dtype None returns the byte size, else a host array of that dtype."""
+def fp_get_tensor(h, what, layer=0, mat=0, dtype=None, count=None):
+    """With dtype None returns the byte size, else a host array of that dtype
+    (its first ``count`` elements when given)."""
     n = _check(_lib.fp_get_tensor(h, what, layer, mat, None, 0), h)
     if dtype is None:
         return n
-    buf = np.empty(n // np.dtype(dtype).itemsize, dtype=dtype)
+    k = n // np.dtype(dtype).itemsize
+    buf = np.empty(k if count is None else min(k, count), dtype=dtype)
     _check(_lib.fp_get_tensor(h, what, layer, mat, _ptr(buf), buf.nbytes), h)
     return buf
 
