@@ -266,6 +266,52 @@ def run_sweep(args):
     return 0
 
 
+# ---------------------------------------------------------------- estimator
+def run_estimate(args, cfg):
+    """L2 / M2 of the paper on this config: fingerprints with 1 and 2 hidden
+    layers at two output lengths -> Eqs. 1-3 -> predicted request latency
+    and footprint of deeper models, next to the measured ones (3, 4 and the
+    full depth of the named model)."""
+    import torch
+
+    import paper_2501_13111_gb300 as fp
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    arch, wq, kvq, B, S, N = cfg
+    full = {"l7b": 32, "l13b": 40, "l70b": 80, "tiny": 4}[args.config]
+    lens = (16, 64)
+
+    def measure(L, n, iters):
+        h = fp.fp_create(arch_dict((L,) + tuple(arch[1:])), wq, kvq, B, S + N + 1, seed=0)
+        try:
+            r = fp.fp_profile(h, S, n, warmup=1, iters=iters)
+            return r.request_ms, r.ttft_ms, r.tpot_ms, r.peak_hbm_bytes
+        finally:
+            fp.fp_destroy(h)
+
+    fits, mem = {}, {}
+    for L in (1, 2):
+        lat = [measure(L, n, 3) for n in lens]
+        fits[L] = fp.fp_solve_eq1(lens[0], lat[0][0], lens[1], lat[1][0])
+        mem[L] = lat[0][3]
+    t = fp.fp_solve_eq23(1, fits[1], 2, fits[2])
+    rows = []
+    for L in (3, 4, full):
+        req, ttft, tpot, peak = measure(L, N, 2)
+        pred = fp.fp_predict_latency(t, L, N)
+        pmem = fp.fp_extrapolate_memory(1, mem[1], 2, mem[2], L)
+        rows.append({"layers": L, "output_length": N, "predicted_ms": pred, "measured_ms": req,
+                     "rel_err": (pred - req) / req, "predicted_ttft_ms": L * t.ttft_layer + t.ttft_other,
+                     "measured_ttft_ms": ttft, "predicted_tpot_ms": L * t.tpot_layer + t.tpot_other,
+                     "measured_tpot_ms": tpot, "predicted_peak_hbm_bytes": pmem, "measured_peak_hbm_bytes": peak})
+    print(json.dumps({"config": config_json(args, cfg), "fits": {L: {"ttft_ms": f.ttft, "tpot_ms": f.tpot}
+                                                                 for L, f in fits.items()},
+                      "terms_ms": {"ttft_layer": t.ttft_layer, "ttft_other": t.ttft_other,
+                                   "tpot_layer": t.tpot_layer, "tpot_other": t.tpot_other},
+                      "checks": rows}), flush=True)
+    return 0
+
+
 # ---------------------------------------------------------------- our arm
 def main():
     ap = argparse.ArgumentParser()
@@ -277,10 +323,13 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass (profiling runs)")
     ap.add_argument("--sweep", action="store_true", help="profile the 96-point configuration sweep instead")
+    ap.add_argument("--estimate", action="store_true", help="run the paper's L2/M2 estimators on --config instead")
     args = ap.parse_args()
     if args.sweep:
         return run_sweep(args)
     cfg = CONFIGS[args.config]
+    if args.estimate:
+        return run_estimate(args, cfg)
     if args.impl == "reference":
         return run_reference(args, cfg)
 

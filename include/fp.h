@@ -75,7 +75,7 @@ typedef struct fp_arch {
   float rope_base; /* e.g. 10000                                           */
 } fp_arch;
 
-#define FP_MAX_LAYERS 8
+#define FP_MAX_LAYERS 80 /* Llama-2-70B depth: the full model runs too */
 
 /* Optional device allocator.  alloc returns a device pointer aligned to at
  * least 256 bytes, or NULL on failure (fp_create then returns FP_ERR_OOM and
@@ -189,6 +189,8 @@ typedef struct fp_profile_result {
   unsigned long long memgetinfo_bytes; /* cudaMemGetInfo drop across fp_create    */
   unsigned long long decode_bytes_per_step; /* algorithmic, at the mean context   */
   int n_layers, prompt_len, n_decode, iters;
+  double request_ms;          /* one request: prefill + n_decode decode steps, device
+                                 events, mean over iters (the latency of Eq. 1) */
 } fp_profile_result;
 
 /* Profile latency and memory: `warmup` untimed passes, then `iters` timed

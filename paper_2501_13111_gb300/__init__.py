@@ -31,7 +31,7 @@ FP_ERR_CUDA, FP_ERR_CAPACITY, FP_ERR_DEVICE_ASSERT, FP_ERR_STATE = -4, -5, -6, -
 FP_W_BF16, FP_W_INT8, FP_W_INT4_G128 = 0, 1, 2
 FP_KV_BF16, FP_KV_INT8 = 0, 1
 FP_FLAG_KEEP_HIDDEN, FP_FLAG_NO_INIT = 1, 2
-FP_MAX_LAYERS = 8
+FP_MAX_LAYERS = 80
 (FP_T_ATTN_NORM, FP_T_WQ, FP_T_WK, FP_T_WV, FP_T_WO, FP_T_FFN_NORM, FP_T_WGATE, FP_T_WUP,
  FP_T_WDOWN) = range(9)
 FP_T_EMBED, FP_T_FINAL_NORM, FP_T_LM_HEAD = 0, 1, 2
@@ -76,7 +76,7 @@ class fp_profile_result(C.Structure):
                 ("weight_bytes", C.c_ulonglong), ("kv_bytes", C.c_ulonglong), ("act_bytes", C.c_ulonglong),
                 ("workspace_bytes", C.c_ulonglong), ("memgetinfo_bytes", C.c_ulonglong),
                 ("decode_bytes_per_step", C.c_ulonglong), ("n_layers", C.c_int), ("prompt_len", C.c_int),
-                ("n_decode", C.c_int), ("iters", C.c_int)]
+                ("n_decode", C.c_int), ("iters", C.c_int), ("request_ms", C.c_double)]
 
     def as_dict(self):
         d = {}
@@ -101,6 +101,15 @@ class fp_kv_view(C.Structure):
                 ("pages_per_seq", C.c_int), ("n_pages", C.c_int), ("k_pool", C.c_void_p),
                 ("v_pool", C.c_void_p), ("k_scale", C.c_void_p), ("v_scale", C.c_void_p),
                 ("page_table", C.c_void_p)]
+
+
+class fp_eq1_fit(C.Structure):
+    _fields_ = [("ttft", C.c_double), ("tpot", C.c_double)]
+
+
+class fp_l2_terms(C.Structure):
+    _fields_ = [("ttft_layer", C.c_double), ("ttft_other", C.c_double), ("tpot_layer", C.c_double),
+                ("tpot_other", C.c_double)]
 
 
 # ------------------------------------------------------------------ prototypes
@@ -134,6 +143,10 @@ _PROTOS = {
     "fp_op_attention_decode_noalloc": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _P]),
     "fp_op_attention_prefill": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P]),
     "fp_op_argmax": (_I, [_P, _I, _I, _P, _P]),
+    "fp_solve_eq1": (_I, [_I, C.c_double, _I, C.c_double, C.POINTER(fp_eq1_fit)]),
+    "fp_solve_eq23": (_I, [_I, C.POINTER(fp_eq1_fit), _I, C.POINTER(fp_eq1_fit), C.POINTER(fp_l2_terms)]),
+    "fp_predict_latency": (_I, [C.POINTER(fp_l2_terms), _I, _I, C.POINTER(C.c_double)]),
+    "fp_extrapolate_memory": (_I, [_I, C.c_double, _I, C.c_double, _I, C.POINTER(C.c_double)]),
 }
 for _name, (_res, _args) in _PROTOS.items():
     _f = getattr(_lib, _name)
@@ -354,3 +367,36 @@ class TorchAllocator:
 
     def _do_free(self, ptr, ctx):
         self.live.pop(ptr, None)
+
+
+# ------------------------------------------------------------------ fp_estimate.h
+def _check_est(code):
+    if code < 0:
+        raise FPError(int(code), "estimator: singular system (equal output lengths or layer counts) or NULL")
+    return code
+
+
+def fp_solve_eq1(len_a, lat_a, len_b, lat_b):
+    """Eq. 1 fitted to two requests of one fingerprint -> fp_eq1_fit (ttft, tpot)."""
+    out = fp_eq1_fit()
+    _check_est(_lib.fp_solve_eq1(len_a, lat_a, len_b, lat_b, C.byref(out)))
+    return out
+
+
+def fp_solve_eq23(layers_a, fit_a, layers_b, fit_b):
+    """Eqs. 2-3 from two fingerprint depths -> fp_l2_terms."""
+    out = fp_l2_terms()
+    _check_est(_lib.fp_solve_eq23(layers_a, C.byref(fit_a), layers_b, C.byref(fit_b), C.byref(out)))
+    return out
+
+
+def fp_predict_latency(terms, num_layers, output_length):
+    v = C.c_double()
+    _check_est(_lib.fp_predict_latency(C.byref(terms), num_layers, output_length, C.byref(v)))
+    return v.value
+
+
+def fp_extrapolate_memory(layers_a, mem_a, layers_b, mem_b, num_layers):
+    v = C.c_double()
+    _check_est(_lib.fp_extrapolate_memory(layers_a, mem_a, layers_b, mem_b, num_layers, C.byref(v)))
+    return v.value

@@ -798,7 +798,7 @@ int fp_profile(fp_handle* h, int prompt_len, int n_decode, int warmup, int iters
   if (e != cudaSuccess) return h->cuda_fail(e, "warmup");
   std::vector<cudaEvent_t> ev((size_t)iters * (n_decode + 2));
   for (auto& x : ev) cudaEventCreate(&x);
-  double ttft = 0, dec = 0;
+  double ttft = 0, dec = 0, req = 0;
   std::vector<double> steps;
   for (int it = 0; it < iters && !st; ++it) {
     cudaEvent_t* E = &ev[(size_t)it * (n_decode + 2)];
@@ -818,6 +818,8 @@ int fp_profile(fp_handle* h, int prompt_len, int n_decode, int warmup, int iters
       float ms = 0;
       cudaEventElapsedTime(&ms, E[0], E[1]);
       ttft += ms;
+      cudaEventElapsedTime(&ms, E[0], E[1 + n_decode]);
+      req += ms;
       for (int j = 0; j < n_decode; ++j) {
         cudaEventElapsedTime(&ms, E[1 + j], E[2 + j]);
         steps.push_back(ms);
@@ -830,6 +832,7 @@ int fp_profile(fp_handle* h, int prompt_len, int n_decode, int warmup, int iters
   if ((st = check_err_flag(h))) return st;
   const fp_arch& a = h->a;
   out->ttft_ms = ttft / iters;
+  out->request_ms = req / iters;
   out->n_layers = a.n_layers;
   out->prompt_len = prompt_len;
   out->n_decode = n_decode;

@@ -10,7 +10,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def _declared():
     names = set()
-    for hdr in ("fp.h", "fp_ops.h"):
+    for hdr in sorted(f for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h")):
         src = open(os.path.join(ROOT, "include", hdr)).read()
         src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
         for m in re.finditer(r"^[A-Za-z_][\w\s\*]*?\b(fp_\w+)\s*\(", src, flags=re.M):
@@ -50,7 +50,7 @@ def _arch(**kw):
 @pytest.mark.parametrize("kw,wq,code", [
     (dict(head_dim=96), 0, -2),
     (dict(n_heads=8, n_kv_heads=3), 0, -1),
-    (dict(n_layers=9), 0, -2),
+    (dict(n_layers=81), 0, -2),
     (dict(hidden=520), 0, -2),
     (dict(ffn=1376), 2, -2),   # int4 needs ffn % 128
     (dict(n_heads=32, n_kv_heads=2), 0, -2),  # group of 16 is not built
