@@ -1,18 +1,19 @@
 // Prefill weight-only linear on the 5th-generation tensor cores.
 //
 // y[M][N] = x[M][K] W[N][K]^T for M > 64 (prefill), the dense contraction of
-// the block's linear layers.  A CTA computes one 128 x 256 output tile over
-// the whole K:
+// the block's linear layers.  One persistent CTA per SM walks 128 x 256
+// output tiles, each over the whole K:
 //   warp 0      TMA producer: x tile [128][64] and W tile [256][64] (bf16,
 //               128-byte swizzled, K-major) into a 4-stage shared ring,
 //               completion counted in bytes on mbarrier full[s];
-//   warp 1      allocates 256 TMEM columns and, from one thread, issues
-//               tcgen05.mma (M 128, N 256, K 16, fp32 accumulation in TMEM);
-//               tcgen05.commit frees each stage (empty[s]) and finally
-//               signals the epilogue;
+//   warp 1      allocates 512 TMEM columns (two fp32 accumulators) and, from
+//               one thread, issues tcgen05.mma (M 128, N 256, K 16);
+//               tcgen05.commit frees each stage (empty[s]) and signals a full
+//               accumulator (tfull[b]);
 //   warps 2-5   epilogue: tcgen05.ld of the accumulator (one TMEM lane per
 //               output row), per-column int8 scale, residual add / SwiGLU /
-//               fp32 store.
+//               fp32 store; then the buffer goes back to the MMA thread
+//               (tempty[b]) while the next tile accumulates in the other.
 // Quantised weights are first expanded to bf16 into a scratch matrix by
 // dequant_kernel (int8: the code itself, exact, with its row scale applied
 // in the epilogue; int4: bf16((q - z) * s)).
@@ -32,7 +33,7 @@ namespace fpk {
 constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64, kTcStages = 4;
 constexpr int kTcThreads = 192;
 constexpr uint32_t kTcStageBytes = (kTcBM + kTcBN) * kTcBK * 2;  // 48 KiB
-constexpr uint32_t kTcTmemCols = 256;
+constexpr uint32_t kTcTmemCols = 512;  // two 256-column fp32 accumulators
 constexpr long long kTcSpinLimit = 1LL << 20;  // try_wait rounds; legit waits here are < 1 ms
 
 // ------------------------------------------------------------------ PTX helpers
@@ -116,13 +117,18 @@ FP_DEV void tc_ld32(uint32_t taddr, float* v) {
 }
 
 // ------------------------------------------------------------------ kernel
+// Persistent: CTA c takes output tiles c, c + gridDim.x, ... in grouped
+// order (16 M tiles share each sweep over the N tiles, so a wave's x rows
+// and weight columns stay in L2).  The shared ring runs across tiles, and
+// the fp32 accumulator is double-buffered in TMEM (2 x 256 columns): the MMA
+// thread fills one buffer while the epilogue warps drain the other.
 // SCALE: multiply output column n by bf16 scales[n] (int8 weights).
 template <int EPI, bool SCALE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int M, int N,
                    int K, const uint16_t* __restrict__ scales, const uint16_t* R, void* Y, int32_t* err) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t full[kTcStages], empty[kTcStages], tmem_full;
+  __shared__ uint64_t full[kTcStages], empty[kTcStages], tfull[2], tempty[2], mma_done;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_word;
   volatile int* abort_flag = &abort_word;  // set by a role that gave up waiting
@@ -132,8 +138,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
   const int Nout = NR == 2 ? N / 2 : N;
   constexpr int BNout = kTcBN / NR;
-  const int n0 = blockIdx.x * BNout, m0 = blockIdx.y * kTcBM;
+  const int tiles_m = (M + kTcBM - 1) / kTcBM, tiles_n = (Nout + BNout - 1) / BNout;
+  const int ntiles = tiles_m * tiles_n;
   const int kblocks = (K + kTcBK - 1) / kTcBK;
+  auto tile_origin = [&](int t, int& m0, int& n0) {
+    constexpr int GM = 16;
+    const int span = GM * tiles_n;
+    const int first = (t / span) * GM;
+    const int gs = min(GM, tiles_m - first);
+    const int r = t % span;
+    m0 = (first + r % gs) * kTcBM;
+    n0 = (r / gs) * BNout;
+  };
 
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -141,7 +157,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(&tmem_full, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);   // tcgen05.commit of the tile's last MMAs
+      mbar_init(&tempty[b], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(&mma_done, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -160,55 +180,90 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   if (warp == 0) {
     // ---------------- TMA producer
     if (lane == 0) {
-      for (int kb = 0; kb < kblocks; ++kb) {
-        const int s = kb % kTcStages;
-        if (!mbar_wait(&empty[s], ((kb / kTcStages) & 1) ^ 1) || *abort_flag) {
-          *abort_flag = 1;
-          if (err) atomicExch(err, 2);
-          break;
-        }
-        uint8_t* a = smem + s * kTcStageBytes;
-        uint8_t* b = a + kTcBM * kTcBK * 2;
-        mbar_expect_tx(&full[s], kTcStageBytes);
-        tma_load_2d(a, &map_x, kb * kTcBK, m0, &full[s]);
-        if (NR == 1) {
-          tma_load_2d(b, &map_w, kb * kTcBK, n0, &full[s]);
-        } else {
-          tma_load_2d(b, &map_w, kb * kTcBK, n0, &full[s]);                              // gate rows
-          tma_load_2d(b + 128 * kTcBK * 2, &map_w, kb * kTcBK, Nout + n0, &full[s]);  // up rows
+      int it = 0;  // k-blocks issued, across tiles
+      for (int t = blockIdx.x; t < ntiles && !*abort_flag; t += gridDim.x) {
+        int m0, n0;
+        tile_origin(t, m0, n0);
+        for (int kb = 0; kb < kblocks; ++kb, ++it) {
+          const int s = it % kTcStages;
+          if (!mbar_wait(&empty[s], ((it / kTcStages) & 1) ^ 1) || *abort_flag) {
+            *abort_flag = 1;
+            if (err) atomicExch(err, 2);
+            break;
+          }
+          uint8_t* a = smem + s * kTcStageBytes;
+          uint8_t* b = a + kTcBM * kTcBK * 2;
+          mbar_expect_tx(&full[s], kTcStageBytes);
+          tma_load_2d(a, &map_x, kb * kTcBK, m0, &full[s]);
+          if (NR == 1) {
+            tma_load_2d(b, &map_w, kb * kTcBK, n0, &full[s]);
+          } else {
+            tma_load_2d(b, &map_w, kb * kTcBK, n0, &full[s]);                              // gate rows
+            tma_load_2d(b + 128 * kTcBK * 2, &map_w, kb * kTcBK, Nout + n0, &full[s]);  // up rows
+          }
         }
       }
+      // copies still in flight land before the CTA leaves (their stages are its shared memory)
+      for (int j = max(0, it - kTcStages); j < it; ++j) mbar_wait(&full[j % kTcStages], (j / kTcStages) & 1);
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = tc_idesc(kTcBM, kTcBN);
-      for (int kb = 0; kb < kblocks; ++kb) {
-        const int s = kb % kTcStages;
-        if (!mbar_wait(&full[s], (kb / kTcStages) & 1) || *abort_flag) {
+      int it = 0, lt = 0;
+      for (int t = blockIdx.x; t < ntiles && !*abort_flag; t += gridDim.x, ++lt) {
+        const int acc = lt & 1;
+        // the epilogue has drained this accumulator (local tile lt - 2)
+        if (!mbar_wait(&tempty[acc], ((lt >> 1) & 1) ^ 1) || *abort_flag) {
           *abort_flag = 1;
           if (err) atomicExch(err, 2);
           break;
         }
         tc_fence_after();
-        const uint32_t a = smem_u32(smem + s * kTcStageBytes);
-        const uint32_t b = a + kTcBM * kTcBK * 2;
+        const uint32_t d = tmem + (uint32_t)acc * kTcBN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb, ++it) {
+          const int s = it % kTcStages;
+          if (!mbar_wait(&full[s], (it / kTcStages) & 1) || *abort_flag) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a = smem_u32(smem + s * kTcStageBytes);
+          const uint32_t b = a + kTcBM * kTcBK * 2;
 #pragma unroll
-        for (int kk = 0; kk < kTcBK / 16; ++kk)
-          tc_mma(tmem, sdesc(a + kk * 32), sdesc(b + kk * 32), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
-        tc_commit(&empty[s]);  // stage s is free once these MMAs have read it
+          for (int kk = 0; kk < kTcBK / 16; ++kk)
+            tc_mma(d, sdesc(a + kk * 32), sdesc(b + kk * 32), idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(&empty[s]);  // stage s is free once these MMAs have read it
+        }
+        if (!ok) {
+          *abort_flag = 1;
+          if (err) atomicExch(err, 2);
+          break;
+        }
+        tc_commit(&tfull[acc]);  // the tile's accumulator is complete
       }
-      tc_commit(&tmem_full);  // all MMAs done (or none, on abort: the barrier still flips)
+      // every MMA issued has completed before TMEM is released
+      tc_commit(&mma_done);
+      mbar_wait(&mma_done, 0);
     }
   } else {
     // ---------------- epilogue: warp w reads TMEM lanes 32 (w % 4) .. +31
     const int q = warp & 3;
-    const int row = m0 + q * 32 + lane;
-    const bool ok = mbar_wait(&tmem_full, 0);
-    if (!ok && err) atomicExch(err, 2);
-    tc_fence_after();
-    if (ok && !*abort_flag) {
-      const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
+    int lt = 0;
+    for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
+      const int acc = lt & 1;
+      int m0, n0;
+      tile_origin(t, m0, n0);
+      const bool ok = mbar_wait(&tfull[acc], (lt >> 1) & 1);
+      if (!ok || *abort_flag) {
+        if (!ok && err) atomicExch(err, 2);
+        *abort_flag = 1;
+        break;
+      }
+      tc_fence_after();
+      const int row = m0 + q * 32 + lane;
+      const uint32_t tl = tmem + (uint32_t)acc * kTcBN + ((uint32_t)(q * 32) << 16);
 #pragma unroll 1
       for (int c0 = 0; c0 < BNout; c0 += 32) {
         float v[32], u[32];
@@ -258,6 +313,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
         }
       }
+      // this warp's reads of the accumulator are done: hand the buffer back to the MMA thread
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(&tempty[acc])) : "memory");
     }
   }
   tc_fence_before();
@@ -348,7 +407,16 @@ static cudaError_t launch_tc_t(const CUtensorMap& mx, const CUtensorMap& mw, int
   }
   const int Nout = EPI == FP_EPI_SWIGLU ? N / 2 : N;
   const int bn = kTcBN / (EPI == FP_EPI_SWIGLU ? 2 : 1);
-  dim3 grid((Nout + bn - 1) / bn, (M + kTcBM - 1) / kTcBM);
+  const long long tiles = (long long)((Nout + bn - 1) / bn) * ((M + kTcBM - 1) / kTcBM);
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        sms <= 0)
+      sms = 152;
+  }
+  // persistent: one CTA per SM (its shared ring and 512 TMEM columns fill the SM)
+  const dim3 grid((unsigned)std::min<long long>(tiles, sms));
   return launch(kern, grid, dim3(kTcThreads), smem, s, mx, mw, M, N, K, scales, R, Y, err);
 }
 
