@@ -33,11 +33,15 @@ static constexpr float kLog2e = 1.4426950408889634f;
 // warps are merged at the end; a second kernel merges the context splits.
 // =====================================================================
 constexpr int kDecTT = 64;  // tokens per tile
-constexpr int kDecNB = 3;   // ring depth
 
+// Ring depth: 3 tiles (two in flight, 2 CTAs per SM with the bf16 cache) when
+// the (sequence, KV head) pairs leave SMs with room, else 2 tiles (one in
+// flight) so that 3 CTAs share an SM -- with pairs to spare, more resident
+// warps beat a deeper ring.
 struct DecodeGeom {
   int chunk;   // positions per split (multiple of kDecTT)
   int splits;  // ceil(max_len / chunk)
+  int nb;      // ring depth
 };
 
 static int dec_sm_count() {
@@ -51,9 +55,10 @@ static int dec_sm_count() {
   return n;
 }
 
-// Resident decode CTAs per SM assumed by the split geometry (the bf16 ring
-// of 104 KB allows two).
-constexpr int kDecOcc = 2;
+// Resident decode CTAs per SM assumed by the split geometry for a ring depth
+// (the bf16 ring takes 104 KB at 3 tiles, 70 KB at 2).
+constexpr int dec_occ(int nb) { return nb == 2 ? 3 : 2; }
+static int dec_ring_depth(long long pairs) { return pairs >= 2LL * dec_sm_count() ? 2 : 3; }
 
 // Split count: the candidates are the counts a whole number of tiles per
 // split produces; each is scored as (waves of resident CTAs) x (tiles per
@@ -67,17 +72,19 @@ constexpr int kDecMaxChunkTiles = 256;  // a split covers at most 16384 position
 static int dec_min_splits(int tiles) { return (tiles + kDecMaxChunkTiles - 1) / kDecMaxChunkTiles; }
 
 static int dec_max_splits(long long pairs, int tiles) {
-  const long long slots = (long long)dec_sm_count() * kDecOcc;
+  const long long slots = (long long)dec_sm_count() * dec_occ(2);  // the larger occupancy bounds both depths
   const long long s = std::max<long long>(std::min(tiles, 4), std::min<long long>(tiles, 2 * slots / std::max<long long>(1, pairs)));
   return (int)std::max<long long>(std::max<long long>(s, 1), dec_min_splits(tiles));
 }
 
 static DecodeGeom decode_geom(int B, int n_kv_heads, int max_len) {
   const long long pairs = (long long)B * n_kv_heads;
-  const long long slots = (long long)dec_sm_count() * kDecOcc;
+  const int nb = dec_ring_depth(pairs);
+  const long long slots = (long long)dec_sm_count() * dec_occ(nb);
   const int tiles = std::max(1, (max_len + kDecTT - 1) / kDecTT);
-  const int smax = dec_max_splits(pairs, tiles);
-  DecodeGeom best{tiles * kDecTT, 1};
+  const int smax = std::min(dec_max_splits(pairs, tiles),
+                            (int)std::max<long long>(std::min<long long>(tiles, 4), 2 * slots / std::max(1LL, pairs)));
+  DecodeGeom best{tiles * kDecTT, 1, nb};
   double best_t = 1e30;
   for (int s = std::max(1, dec_min_splits(tiles)); s <= smax; ++s) {
     const int per = (tiles + s - 1) / s;
@@ -162,31 +169,31 @@ FP_DEV uint2 dec_i8_to_f16x4(uint32_t w) {
   return make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&b));
 }
 
-template <int HD, int KVQ>
+template <int HD, int KVQ, int NB>
 constexpr size_t dec_smem_bytes() {
   constexpr size_t ld = HD + 8;  // padded 16-bit row (elements)
-  if (KVQ == FP_KV_BF16) return (size_t)kDecNB * kDecTT * ld * 2 * 2;
+  if (KVQ == FP_KV_BF16) return (size_t)NB * kDecTT * ld * 2 * 2;
   // int8: ring of code rows (HD + 16 bytes), per-token scales, one fp16 tile of K and V
-  return (size_t)kDecNB * kDecTT * (HD + 16) * 2 + (size_t)kDecNB * kDecTT * 2 * sizeof(float) +
+  return (size_t)NB * kDecTT * (HD + 16) * 2 + (size_t)NB * kDecTT * 2 * sizeof(float) +
          (size_t)kDecTT * ld * 2 * 2;
 }
 
 // The ring, which also holds the 4-warp merge buffer after the loop; the
 // chunk's page ids follow it.
-template <int HD, int KVQ, int G>
+template <int HD, int KVQ, int G, int NB>
 constexpr size_t dec_stage_bytes() {
-  return std::max(dec_smem_bytes<HD, KVQ>(), (size_t)4 * G * (HD + 2) * sizeof(float));
+  return std::max(dec_smem_bytes<HD, KVQ, NB>(), (size_t)4 * G * (HD + 2) * sizeof(float));
 }
 
 // Workspace layout for (b, h, split): o [HD] fp32 (un-normalised, relative to
 // m), then (m, l) in the log2 domain.
-template <int HD, int KVQ, int G>
+template <int HD, int KVQ, int G, int NB>
 __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __restrict__ q, int q_stride, int H,
                                                           fp_kv_view kv, const int32_t* __restrict__ len,
                                                           int len_add, int max_len, int chunk, int splits,
                                                           float* __restrict__ ws, uint16_t* __restrict__ out,
                                                           int32_t* err) {
-  constexpr int TT = kDecTT, NB = kDecNB, LD = HD + 8;
+  constexpr int TT = kDecTT, LD = HD + 8;
   constexpr bool I8 = KVQ == FP_KV_INT8;
   constexpr int RAWB = I8 ? HD + 16 : LD * 2;  // bytes per staged row
   constexpr int CPR = (I8 ? HD : HD * 2) / 16;  // 16-byte chunks per row
@@ -220,7 +227,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const uint16_t* __rest
   const int ntile = (t1 - t0 + TT - 1) / TT;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // ---- the page ids of positions t0 .. t1-1, staged once (past the table: -1)
-  int* spt = reinterpret_cast<int*>(smem + dec_stage_bytes<HD, KVQ, G>());
+  int* spt = reinterpret_cast<int*>(smem + dec_stage_bytes<HD, KVQ, G, NB>());
   {
     const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
     const int lp0 = t0 / kv.page_size, n = (t1 - 1) / kv.page_size - lp0 + 1;
@@ -467,13 +474,13 @@ __global__ void attn_combine_kernel(int H, const int32_t* __restrict__ len, int 
   out[(long long)bh * HD + e] = f2bf(o / L);
 }
 
-template <int HD, int KVQ, int G>
-static cudaError_t launch_decode_t(const uint16_t* q, int q_stride, int B, int H, const fp_kv_view& kv,
-                                   const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
-                                   uint16_t* out, int32_t* err, cudaStream_t s, cudaError_t* second) {
+template <int HD, int KVQ, int G, int NB>
+static cudaError_t launch_decode_nb(const uint16_t* q, int q_stride, int B, int H, const fp_kv_view& kv,
+                                    const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
+                                    uint16_t* out, int32_t* err, cudaStream_t s, cudaError_t* second) {
   // the ring also holds the 4-warp merge buffer after the loop
-  const size_t smem = dec_stage_bytes<HD, KVQ, G>() + ((size_t)g.chunk / kv.page_size + 2) * sizeof(int);
-  auto kern = attn_decode_kernel<HD, KVQ, G>;
+  const size_t smem = dec_stage_bytes<HD, KVQ, G, NB>() + ((size_t)g.chunk / kv.page_size + 2) * sizeof(int);
+  auto kern = attn_decode_kernel<HD, KVQ, G, NB>;
   if (smem > 48 * 1024) FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   dim3 grid(B * kv.n_kv_heads, g.splits);
   cudaError_t e = launch(kern, grid, dim3(128), smem, s, q, q_stride, H, kv, len, len_add, max_len, g.chunk,
@@ -483,6 +490,14 @@ static cudaError_t launch_decode_t(const uint16_t* q, int q_stride, int B, int H
              (const float*)ws, out);
   if (second) *second = e;
   return e;
+}
+
+template <int HD, int KVQ, int G>
+static cudaError_t launch_decode_t(const uint16_t* q, int q_stride, int B, int H, const fp_kv_view& kv,
+                                   const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
+                                   uint16_t* out, int32_t* err, cudaStream_t s, cudaError_t* second) {
+  return g.nb == 2 ? launch_decode_nb<HD, KVQ, G, 2>(q, q_stride, B, H, kv, len, len_add, max_len, g, ws, out, err, s, second)
+                   : launch_decode_nb<HD, KVQ, G, 3>(q, q_stride, B, H, kv, len, len_add, max_len, g, ws, out, err, s, second);
 }
 
 template <int HD, int KVQ>
