@@ -1,0 +1,513 @@
+// Decode linear for int4 group-128 weights at 17-64 tokens on the tcgen05
+// tensor cores.
+//
+// y[m][n] = sum_k x[m][k] (q[n][k] - z[n][g]) s[n][g], g = k / 128, the
+// weight-only linear of a decoder block (QKV, O, gate+up, down) while the
+// decode batch is large enough that int4 dequantisation plus the legacy
+// mma.sync rate, not HBM, bound the CUDA-core GEMV (two weights per byte,
+// 2 M flop per weight).  The weights are the A operand (128 rows, one TMEM
+// lane each) and the tokens the N dimension of tcgen05.mma (M 128, N =
+// tokens rounded up to 32 or 64, K 16):
+//   warps 0-15  dequantise, in two teams of eight that take alternate
+//               128-k groups: warp w owns TMEM lanes 32 (w % 4) .. +31 (one
+//               weight row per thread) and half of a group (SwiGLU: a whole
+//               group of the gate or the up tile).  Each thread streams its
+//               own codes through a private cp.async ring in shared memory
+//               (no cross-warp handshake),
+//               forms bf16((q - z) s) -- exactly the prefill expansion --
+//               and stores them into an A slot of TMEM (tcgen05.st, two K
+//               elements per 32-bit column); afull / aempty hand the slots
+//               to the MMA thread and back;
+//   warp 16     TMA producer of x ([N][128] bf16 per group, two
+//               128-byte-swizzled boxes, rows past M zero-filled) into a ring
+//               (xfull / xempty, freed by the MMAs);
+//   warp 17     allocates 512 TMEM columns and issues the MMAs (A from TMEM,
+//               B = x from shared memory) into fp32 TMEM accumulators.
+// MMAs (M 128, N <= 64, K 16) into one accumulator follow each other at
+// about 50 cycles, far above their math (N / 2 cycles), while MMAs into
+// different accumulators overlap: the k-steps of each matrix are spread
+// round-robin over 2-4 accumulators ("chains"), summed in the epilogue.
+// The (row tile, group) pairs are split into equal contiguous ranges, one
+// per SM (stream-K, as the CUDA-core GEMV): a CTA whose range covers a whole
+// row tile runs the epilogue itself; otherwise each of its sixteen warps
+// writes fp32 partials of its 32 rows x a quarter of the tokens, and the
+// last CTA to finish that slice (a ticket per slice) sums them in CTA order
+// and runs the epilogue -- residual add, SwiGLU, bf16 or fp32 store.
+//
+// Every mbarrier wait is bounded; past the limit the thread records error 2
+// in the error word, the CTA stops and releases TMEM after its copies and
+// MMAs have completed.
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.cuh"
+#include "tc.cuh"
+
+namespace fpk {
+
+constexpr int kQ4CodeStages = 4;  // per-thread cp.async ring depth, one (own) group per stage
+constexpr int kQ4DeqWarps = 16;
+constexpr int kQ4MmaWarps = 2;  // MMA issuers, each with its own accumulators
+constexpr int kQ4Threads = (kQ4DeqWarps + 1 + kQ4MmaWarps) * 32;
+constexpr uint32_t kQ4TmemCols = 512;
+constexpr int kQ4Rows = 128;
+constexpr int kQ4MinSmem = 116 * 1024;  // above half an SM: one CTA (and one TMEM owner) per SM
+
+template <int MT, int NR>
+struct Q4Geom {
+  // each thread takes every other group: a whole group of its row (SwiGLU:
+  // of the gate or the up row), otherwise half of one
+  static constexpr int kChunks = NR == 2 ? 4 : 2;        // 16-byte code chunks per thread and group
+  static constexpr int kCodeBytes = kQ4DeqWarps * 32 * kChunks * 16;  // one ring stage, all threads
+  static constexpr int kXBytes = MT * 256;               // x [MT][128] bf16 as two [MT][64] boxes
+  // independent accumulation chains per matrix
+  static constexpr int kChains = MT == 64 ? 2 / NR : 4 / NR;
+  static constexpr int kDCols = NR * kChains * MT;       // fp32 accumulators
+  static constexpr int kACols = NR * 64;                 // one group of bf16 pairs per matrix
+  static constexpr int kASlots = std::min(6, ((int)kQ4TmemCols - kDCols) / kACols);
+  static constexpr int kXStages = MT == 64 ? 4 : 6;
+  static constexpr int kSmem = kQ4CodeStages * kCodeBytes + kXStages * kXBytes + 1024;
+  static_assert(kASlots >= 2 && kDCols + kASlots * kACols <= (int)kQ4TmemCols, "TMEM budget");
+  static_assert(kCodeBytes % 1024 == 0 && kXBytes % 1024 == 0, "x stages stay 1024-byte aligned");
+};
+
+// 16-byte asynchronous global -> shared copy (L2 only) and its group fences.
+FP_DEV void q4_cp16(void* smem, const void* gmem) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem) : "memory");
+}
+FP_DEV void q4_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+FP_DEV void q4_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// V consecutive bf16 (V = 8, 4, 2 or 1, aligned to V elements) in a uint4.
+FP_DEV uint4 ld_groups(const uint16_t* p, int V) {
+  if (V == 8) return __ldg(reinterpret_cast<const uint4*>(p));
+  if (V == 4) {
+    const uint2 t = __ldg(reinterpret_cast<const uint2*>(p));
+    return make_uint4(t.x, t.y, 0u, 0u);
+  }
+  if (V == 2) return make_uint4(__ldg(reinterpret_cast<const unsigned int*>(p)), 0u, 0u, 0u);
+  return make_uint4((uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p)), 0u, 0u, 0u);
+}
+
+FP_DEV uint32_t bf16_at(const uint4& v, int j) {
+  const int w = j >> 1;
+  const uint32_t x = w == 0 ? v.x : w == 1 ? v.y : w == 2 ? v.z : v.w;
+  return (j & 1) ? (x >> 16) : (x & 0xFFFFu);
+}
+
+union Bf2 {
+  uint32_t u;
+  __nv_bfloat162 h;
+};
+
+// One packed word of int4 codes (elements 8j .. 8j+7; nibbles i and i + 4
+// hold elements 2i and 2i + 1) -> four bf16 pairs (q - z) s in element order.
+// bf16(128 + q) is formed exactly by the exponent trick; subtracting
+// bf16(128 + z) is exact for integer z in [0, 15]; the product is rounded
+// once, to nearest even.
+FP_DEV void deq_word(uint32_t w, uint32_t zz, uint32_t ss, uint32_t* out) {
+  Bf2 z2, s2;
+  z2.u = zz;
+  s2.u = ss;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    Bf2 p;
+    p.u = ((w >> (4 * i)) & 0x000F000Fu) | 0x43004300u;
+    p.h = __hmul2(__hsub2(p.h, z2.h), s2.h);
+    out[i] = p.u;
+  }
+}
+
+FP_DEV long long q4_cta_of(long long i, long long C, long long total) { return ((i + 1) * C - 1) / total; }
+
+template <int MT, int EPI>
+__global__ void __launch_bounds__(kQ4Threads, 1)
+    gemv_q4tc_kernel(const __grid_constant__ CUtensorMap map_x, const uint8_t* __restrict__ codes, int M, int N,
+                     const uint16_t* __restrict__ scales, const uint16_t* __restrict__ zeros, const uint16_t* R,
+                     void* Y, long long total, int S, int V, float* __restrict__ ws, unsigned* __restrict__ counters,
+                     int32_t* err) {
+  constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
+  using G = Q4Geom<MT, NR>;
+  constexpr int CS = kQ4CodeStages, XS = G::kXStages, NA = G::kASlots, MQ = MT / 4, DW = kQ4DeqWarps;
+  constexpr int NCH = G::kChains, CK = G::kChunks;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  __shared__ uint64_t xfull[XS], xempty[XS], afull[NA], aempty[NA], dfull, dempty, mma_done;
+  __shared__ uint32_t tmem_base;
+  __shared__ int abort_word;
+  volatile int* abort_flag = &abort_word;
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* x_ring = smem;                               // 1024-byte aligned for the 128-byte swizzle
+  uint8_t* code_ring = smem + XS * G::kXBytes;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Nout = NR == 2 ? N / 2 : N;
+  const long long C = gridDim.x, c = blockIdx.x;
+  const long long begin = c * total / C, end = (c + 1) * total / C;
+  const int L = (int)(end - begin);
+  auto fail = [&]() {
+    *abort_flag = 1;
+    if (err) atomicExch(err, 2);
+  };
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < XS; ++s) {
+      mbar_init(&xfull[s], 1);   // producer's expect_tx; completes with the bytes
+      mbar_init(&xempty[s], kQ4MmaWarps);  // tcgen05.commit of the MMAs that read x
+    }
+    for (int a = 0; a < NA; ++a) {
+      mbar_init(&afull[a], DW / 2);  // the eight warps of the group's team stored its A columns
+      mbar_init(&aempty[a], kQ4MmaWarps);  // tcgen05.commit of the MMAs that read the slot
+    }
+    mbar_init(&dfull, kQ4MmaWarps);
+    mbar_init(&dempty, DW);
+    mbar_init(&mma_done, kQ4MmaWarps);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == DW + 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&tmem_base)),
+                 "r"(kQ4TmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = tmem_base;
+
+  if (warp == DW) {
+    // ---------------- TMA producer of x
+    if (lane == 0) {
+      pdl_wait();  // x is the previous kernel's output
+      int issued = 0;
+      int g = (int)(begin % S);
+      for (int q = 0; q < L; ++q, g = g + 1 == S ? 0 : g + 1) {
+        const int s = q % XS;
+        if (q >= XS && (!mbar_wait(&xempty[s], ((q / XS) & 1) ^ 1) || *abort_flag)) {
+          fail();
+          break;
+        }
+        uint8_t* xs = x_ring + s * G::kXBytes;
+        mbar_expect_tx(&xfull[s], G::kXBytes);
+        tma_load_2d(xs, &map_x, g * 128, 0, &xfull[s]);
+        tma_load_2d(xs + MT * 128, &map_x, g * 128 + 64, 0, &xfull[s]);
+        issued = q + 1;
+      }
+      // copies still in flight land before the CTA leaves (their stages are its shared memory)
+      for (int j = max(0, issued - XS); j < issued; ++j) mbar_wait(&xfull[j % XS], (j / XS) & 1);
+    }
+  } else if (warp > DW) {
+    // ---------------- MMA issuers: SwiGLU, one per matrix; otherwise even / odd k-steps
+    const int mw = warp - DW - 1;
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc_idesc(kQ4Rows, MT);
+      int seg = 0;
+      bool ok = true;
+      int g = (int)(begin % S);
+      for (int q = 0; q < L; ++q, g = g + 1 == S ? 0 : g + 1) {
+        const bool first = q == 0 || g == 0, last = g == S - 1 || q == L - 1;
+        const int s = q % XS, a = q % NA;
+        if (first && seg > 0) ok = mbar_wait(&dempty, (seg - 1) & 1);  // the epilogue has read D
+        ok = ok && mbar_wait(&xfull[s], (q / XS) & 1) && mbar_wait(&afull[a], (q / NA) & 1) && !*abort_flag;
+        if (!ok) break;
+        tc_fence_after();
+        const uint64_t xd = sdesc(smem_u32(x_ring + s * G::kXBytes));
+        const uint32_t ta = tmem + G::kDCols + a * G::kACols;
+        // k-step kk of matrix r goes to chain kk % NCH of that matrix: consecutive
+        // MMAs of one issuer never share an accumulator, and the two issuers'
+        // chains are disjoint
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+          const int r = NR == 2 ? mw : 0;
+          if (NR == 1 && (kk & 1) != mw) continue;
+          // descriptor start addresses count 16-byte units
+          tc_mma_ts(tmem + (r * NCH + kk % NCH) * MT, ta + r * 64 + kk * 8,
+                    xd + (uint64_t)(((kk >> 2) * MT * 128 + (kk & 3) * 32) >> 4), idesc, (first && kk < NCH) ? 0u : 1u);
+        }
+        tc_commit(&xempty[s]);  // x of stage s has been read
+        tc_commit(&aempty[a]);  // A slot a has been read
+        if (last) {
+          tc_commit(&dfull);
+          ++seg;
+        }
+      }
+      if (!ok) fail();
+      // every MMA issued has completed before TMEM is released
+      tc_commit(&mma_done);
+      mbar_wait(&mma_done, 0);
+    }
+  } else {
+    // ---------------- dequantise (+ epilogue)
+    // two teams of eight warps take alternate groups, so one team computes
+    // while the other waits; within a team warp w owns TMEM lanes
+    // 32 (w % 4) .. +31 and, SwiGLU, the gate or the up rows, otherwise the
+    // first or second half of the group
+    const int qd = warp & 3, team = warp >> 3, half = (warp >> 2) & 1, lr = qd * 32 + lane;
+    const int pt = warp >> 2;  // epilogue: tokens [pt MQ, (pt + 1) MQ)
+    const int rm = NR == 2 ? half : 0;
+    const int cbase = NR == 2 ? 0 : 2 * half;  // first 16-byte chunk of the row's 64 bytes
+    const int acol = NR == 2 ? rm * 64 : half * 32;
+    const uint32_t lane_base = tmem + ((uint32_t)(qd * 32) << 16);
+    const long long row_bytes = (long long)S * 64;
+
+    // ---- this thread's code ring: its n-th own group (pair team + 2 n) in stage n % CS
+    uint8_t* my_ring = code_ring + (size_t)threadIdx.x * CK * 16;
+    const int own = (L - team + 1) / 2;  // groups this team takes
+    int ib = (int)((begin + team) / S), ig = (int)((begin + team) % S);  // (row tile, group) of the next copy
+    const uint8_t* src = nullptr;
+    auto set_src = [&]() {
+      const long long rr = min(ib * kQ4Rows + lr, Nout - 1) + rm * Nout;
+      src = codes + rr * row_bytes + cbase * 16;
+    };
+    if (own > 0) set_src();
+    auto issue = [&](int n) {  // called for n = 0, 1, 2, ... in order
+      if (n < own) {
+        uint8_t* d = my_ring + (size_t)(n % CS) * G::kCodeBytes;
+#pragma unroll
+        for (int i = 0; i < CK; ++i) q4_cp16(d + i * 16, src + (long long)ig * 64 + i * 16);
+        ig += 2;
+        if (ig >= S) {
+          while (ig >= S) ig -= S, ++ib;
+          if (n + 1 < own) set_src();
+        }
+      }
+      q4_commit();
+    };
+    // the weights are constant: the first stages go out before the previous kernel ends
+#pragma unroll 1
+    for (int n = 0; n < CS - 1; ++n) issue(n);
+
+    // scales and zeros of the row, V groups per load, one chunk ahead (S % V == 0,
+    // so a chunk never crosses a row tile)
+    uint4 s_cur, z_cur, s_nxt = make_uint4(0u, 0u, 0u, 0u), z_nxt = s_nxt;
+    auto load_chunk = [&](int bb, int g0, uint4& sv, uint4& zv) {
+      const long long idx = (long long)(min(bb * kQ4Rows + lr, Nout - 1) + rm * Nout) * S + g0;
+      sv = ld_groups(scales + idx, V);
+      zv = ld_groups(zeros + idx, V);
+    };
+    // (row tile, group) of the current pair and its place j in the chunk of V
+    // groups, advanced without divisions
+    int b = (int)(begin / S), g = (int)(begin % S), j = g % V;
+    load_chunk(b, g - j, s_cur, z_cur);
+    auto prefetch_next = [&](long long p_next, int bb, int g0) {  // the chunk starting at pair p_next
+      if (g0 == S) g0 = 0, ++bb;
+      if (p_next < end) load_chunk(bb, g0, s_nxt, z_nxt);
+    };
+    prefetch_next(begin - j + V, b, g - j + V);
+    pdl_wait();
+    int seg = 0;
+    for (int q = 0; q < L; ++q) {
+      const long long p = begin + q;
+      if (q > 0) {
+        if (++g == S) g = 0, ++b;
+        if (++j == V) {
+          j = 0;
+          s_cur = s_nxt;
+          z_cur = z_nxt;
+          prefetch_next(p + V, b, g + V);
+        }
+      }
+      const bool last = g == S - 1 || q == L - 1;
+      if ((q & 1) == team) {
+        const int n = q >> 1, a = q % NA;
+        q4_wait<CS - 2>();  // this thread's copies of its n-th group have landed
+        uint4 wv[CK];
+#pragma unroll
+        for (int i = 0; i < CK; ++i)
+          wv[i] = *reinterpret_cast<const uint4*>(my_ring + (size_t)(n % CS) * G::kCodeBytes + i * 16);
+        issue(n + CS - 1);  // refills the stage read one own group ago
+
+        const uint32_t sb = bf16_at(s_cur, j);
+        const uint32_t zb = f2bf(128.f + bf2f((uint16_t)bf16_at(z_cur, j)));
+        const uint32_t ss = sb | (sb << 16), zz = zb | (zb << 16);
+        bool ok = mbar_wait_sleep(&aempty[a], ((q / NA) & 1) ^ 1);
+        if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
+          if (lane == 0) fail();
+          break;
+        }
+        tc_fence_after();
+        const uint32_t ta = lane_base + G::kDCols + a * G::kACols + acol;
+#pragma unroll
+        for (int h2 = 0; h2 < CK / 2; ++h2) {  // 32 columns (two chunks) per store
+          uint32_t av[32];
+#pragma unroll
+          for (int i = 0; i < 2; ++i) {
+            const uint4 w = wv[2 * h2 + i];
+            deq_word(w.x, zz, ss, av + i * 16);
+            deq_word(w.y, zz, ss, av + i * 16 + 4);
+            deq_word(w.z, zz, ss, av + i * 16 + 8);
+            deq_word(w.w, zz, ss, av + i * 16 + 12);
+          }
+          tc_st32(ta + h2 * 32, av);
+        }
+        tc_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&afull[a]);
+      }
+      if (!last) continue;
+
+      // ---- the CTA's part of row tile b is accumulated: this warp takes tokens [m0, m0 + MQ)
+      bool ok = mbar_wait_sleep(&dfull, seg & 1);
+      if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
+        if (lane == 0) fail();
+        break;
+      }
+      tc_fence_after();
+      const int m0 = pt * MQ;
+      uint32_t dv[NR][MQ];
+#pragma unroll
+      for (int r = 0; r < NR; ++r) {
+        tc_ld<MQ>(lane_base + r * NCH * MT + m0, dv[r]);
+#pragma unroll
+        for (int ch = 1; ch < NCH; ++ch) {  // the chains' sum, in chain order
+          uint32_t e[MQ];
+          tc_ld<MQ>(lane_base + (r * NCH + ch) * MT + m0, e);
+#pragma unroll
+          for (int i = 0; i < MQ; ++i) dv[r][i] = __float_as_uint(__uint_as_float(dv[r][i]) + __uint_as_float(e[i]));
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&dempty);
+      ++seg;
+
+      const int row = b * kQ4Rows + lr;
+      auto finish = [&](int m, float v, float u) {
+        const long long o = (long long)m * Nout + row;
+        if constexpr (EPI == FP_EPI_STORE) ((uint16_t*)Y)[o] = f2bf(v);
+        else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(bf2f(R[o]) + v);
+        else if constexpr (EPI == FP_EPI_SWIGLU) ((uint16_t*)Y)[o] = f2bf(silu(v) * u);
+        else ((float*)Y)[o] = v;
+      };
+      const long long c0 = q4_cta_of((long long)b * S, C, total);
+      const long long c1 = q4_cta_of((long long)(b + 1) * S - 1, C, total);
+      if (c0 == c1) {
+#pragma unroll
+        for (int i = 0; i < MQ; ++i)
+          if (m0 + i < M && row < Nout) finish(m0 + i, __uint_as_float(dv[0][i]), __uint_as_float(dv[NR - 1][i]));
+        continue;
+      }
+      // partial slot b + c: distinct for every (row tile, CTA) pair that meets
+      const size_t slot = (size_t)M * NR * kQ4Rows;
+      float* part = ws + (size_t)(b + c) * slot;
+#pragma unroll
+      for (int i = 0; i < MQ; ++i)
+        if (m0 + i < M)
+#pragma unroll
+          for (int r = 0; r < NR; ++r) part[((size_t)(m0 + i) * NR + r) * kQ4Rows + lr] = __uint_as_float(dv[r][i]);
+      __threadfence();
+      __syncwarp();
+      unsigned t = 0;
+      if (lane == 0) t = atomicAdd(&counters[b * DW + warp], 1u);
+      t = __shfl_sync(0xffffffffu, t, 0);
+      if (t != (unsigned)(c1 - c0)) continue;
+      __threadfence();
+      const int cnt = (int)(c1 - c0) + 1;
+      for (int i = 0; i < MQ && m0 + i < M; ++i) {
+        const float* p0 = ws + (size_t)(b + c0) * slot + (size_t)(m0 + i) * NR * kQ4Rows + lr;
+        float v = 0.f, u = 0.f;
+        for (int cc = 0; cc < cnt; ++cc) {
+          v += __ldcg(p0 + (size_t)cc * slot);
+          if (NR == 2) u += __ldcg(p0 + (size_t)cc * slot + kQ4Rows);
+        }
+        if (row < Nout) finish(m0 + i, v, u);
+      }
+      if (lane == 0) counters[b * DW + warp] = 0u;
+    }
+    q4_wait<0>();  // copies in flight land before the CTA leaves
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == DW + 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kQ4TmemCols) : "memory");
+  }
+}
+
+// ---------------------------------------------------------------- host side
+static int q4_sms() {
+  static int n = 0;
+  if (!n) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        n <= 0)
+      n = 152;
+  }
+  return n;
+}
+
+static int q4_mt(int M) { return M <= 32 ? 32 : 64; }
+static int q4_v(int groups) { return groups % 8 == 0 ? 8 : groups % 4 == 0 ? 4 : groups % 2 == 0 ? 2 : 1; }
+
+bool q4tc_ok(int wquant, int epi, int M, int N, int K) {
+  if (wquant != FP_W_INT4_G128 || M < 17 || M > 64 || N < 1 || K < 128 || K % 128 != 0) return false;
+  if (epi == FP_EPI_SWIGLU && N % 2 != 0) return false;
+  const long long nout = epi == FP_EPI_SWIGLU ? N / 2 : N;
+  const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
+  return blocks * kQ4DeqWarps <= kLinTicketSlots && tensor_maps_available();
+}
+
+size_t q4tc_ws_bytes(int epi, int M, int N, int K) {
+  const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
+  const long long nout = nr == 2 ? N / 2 : N;
+  const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
+  const long long ctas = std::min<long long>(blocks * (K / 128), q4_sms());
+  return (size_t)kLinTicketSlots * 4 + (size_t)(blocks + ctas) * M * nr * kQ4Rows * 4;
+}
+
+template <int MT, int EPI>
+static cudaError_t launch_q4_t(const uint8_t* codes, const CUtensorMap& mx, int M, int N, int K,
+                               const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* Y, void* ws,
+                               int32_t* err, cudaStream_t s) {
+  constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
+  auto kern = gemv_q4tc_kernel<MT, EPI>;
+  const int smem = std::max(Q4Geom<MT, NR>::kSmem, kQ4MinSmem);
+  static bool attr = false;
+  if (!attr) {
+    FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    attr = true;
+  }
+  const int nout = NR == 2 ? N / 2 : N;
+  const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
+  const int S = K / 128;
+  const long long total = blocks * S;
+  const int ctas = (int)std::min<long long>(total, q4_sms());
+  unsigned* counters = (unsigned*)ws;
+  float* part = (float*)((char*)ws + (size_t)kLinTicketSlots * 4);
+  return launch(kern, dim3(ctas), dim3(kQ4Threads), (size_t)smem, s, mx, codes, M, N, scales, zeros, R, Y, total, S,
+                q4_v(S), part, counters, err);
+}
+
+template <int MT>
+static cudaError_t launch_q4_m(int epi, const uint8_t* mw, const CUtensorMap& mx, int M, int N, int K,
+                               const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* Y, void* ws,
+                               int32_t* err, cudaStream_t s) {
+  switch (epi) {
+    case FP_EPI_STORE: return launch_q4_t<MT, FP_EPI_STORE>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    case FP_EPI_RESID: return launch_q4_t<MT, FP_EPI_RESID>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    case FP_EPI_SWIGLU: return launch_q4_t<MT, FP_EPI_SWIGLU>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    default: return launch_q4_t<MT, FP_EPI_F32>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+  }
+}
+
+cudaError_t launch_q4tc(int epi, const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
+                        const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
+                        int32_t* err, cudaStream_t s) {
+  if (!q4tc_ok(FP_W_INT4_G128, epi, M, N, K)) return cudaErrorInvalidValue;
+  if (!ws || ws_bytes < q4tc_ws_bytes(epi, M, N, K)) return cudaErrorInvalidValue;
+  CUtensorMap mx;
+  const int mt = q4_mt(M);
+  const uint8_t* mw = (const uint8_t*)codes;
+  // x [M][K] bf16, box [mt rows][64]
+  if (!make_tensor_map(&mx, x, M, K, 2, mt, 64, 128)) return cudaErrorInvalidValue;
+  switch (mt) {
+    case 32: return launch_q4_m<32>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s);
+    default: return launch_q4_m<64>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s);
+  }
+}
+
+}  // namespace fpk

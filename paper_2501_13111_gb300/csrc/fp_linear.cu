@@ -591,7 +591,7 @@ static int mma_kt(int wq) { return wq == FP_W_BF16 ? 8 : wq == FP_W_INT8 ? 16 : 
 // Workspace = a fixed area of ticket counters (zero at rest), then the fp32
 // partials.  The ticket area has the same size for every launch, so the
 // partials of one launch never land on the counters of the next.
-constexpr int kTicketSlots = 4096;
+constexpr int kTicketSlots = kLinTicketSlots;
 static size_t counter_bytes(int) { return (size_t)kTicketSlots * 4; }
 
 // One ticket per 128-row block.
@@ -792,8 +792,14 @@ size_t linear_ws_bytes(int wquant, int M, int N, int K) {
   }
   if (!mma_ok(wquant, M, N, K)) return 0;
   size_t w = 0;
-  for (int epi : {FP_EPI_STORE, FP_EPI_RESID, FP_EPI_F32}) w = std::max(w, plan_for(wquant, epi, M, N, K).ws);
-  if (N % 2 == 0) w = std::max(w, plan_for(wquant, FP_EPI_SWIGLU, M, N, K).ws);
+  for (int epi : {FP_EPI_STORE, FP_EPI_RESID, FP_EPI_F32}) {
+    w = std::max(w, plan_for(wquant, epi, M, N, K).ws);
+    if (q4tc_ok(wquant, epi, M, N, K)) w = std::max(w, q4tc_ws_bytes(epi, M, N, K));
+  }
+  if (N % 2 == 0) {
+    w = std::max(w, plan_for(wquant, FP_EPI_SWIGLU, M, N, K).ws);
+    if (q4tc_ok(wquant, FP_EPI_SWIGLU, M, N, K)) w = std::max(w, q4tc_ws_bytes(FP_EPI_SWIGLU, M, N, K));
+  }
   return w;
 }
 
@@ -815,6 +821,9 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
     return launch_gemm_tc(wquant, epi, x, M, N, K, codes, scales, zeros, residual, y, scratch,
                           need ? ws_bytes - counter_bytes(0) : 0, err, s);
   }
+  // int4 at 9-64 tokens: the tensor-core path (TMA needs 16-byte aligned x and codes)
+  if (q4tc_ok(wquant, epi, M, N, K) && ((uintptr_t)x & 15) == 0 && ((uintptr_t)codes & 15) == 0)
+    return launch_q4tc(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, err, s);
   if (mma_ok(wquant, M, N, K)) {
     switch (wquant) {
       case FP_W_BF16: return launch_mma<FP_W_BF16>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s);

@@ -38,6 +38,8 @@ cudaError_t launch_attention_prefill(const uint16_t* q, int q_stride, int B, int
                                      const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s);
 
 // ---- weight-only linear (fp_linear.cu)
+// Split-K ticket counters at the head of a linear's workspace (zero at rest).
+constexpr int kLinTicketSlots = 4096;
 // Workspace of one launch with exactly these M, N, K (any epilogue); 0 if none.
 size_t linear_ws_bytes(int wquant, int M, int N, int K);
 // Largest workspace over every M in [1, max_m].
@@ -45,6 +47,13 @@ size_t linear_ws_bytes_upto(int wquant, int max_m, int N, int K);
 cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
                           void* ws, size_t ws_bytes, cudaStream_t s, int32_t* err = nullptr);
+
+// ---- int4 decode linear at 9-64 tokens on tcgen05 (fp_gemv_tc.cu)
+bool q4tc_ok(int wquant, int epi, int M, int N, int K);
+size_t q4tc_ws_bytes(int epi, int M, int N, int K);
+cudaError_t launch_q4tc(int epi, const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
+                        const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
+                        int32_t* err, cudaStream_t s);
 
 // ---- prefill GEMM on tcgen05 (fp_gemm_tc.cu)
 bool gemm_tc_ok(int M, int N, int K);

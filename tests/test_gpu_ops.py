@@ -118,6 +118,47 @@ def test_linear_long_k(fp, wq, m, n, k):
     assert rel_err(got, ref) <= TAU[wq] / 4, (wq, m, n, k, rel_err(got, ref))
 
 
+@pytest.mark.parametrize("m,n,k,epi", [
+    (9, 200, 1024, 3), (16, 384, 5120, 2), (17, 300, 4096, 1), (32, 1000, 8192, 0), (33, 256, 1152, 3),
+    (48, 520, 2048, 2), (64, 136, 11008, 1), (32, 2048, 3584, 3), (16, 40960, 256, 0), (24, 40960, 256, 2),
+    (17, 1152, 1152, 0)])
+def test_linear_int4_tensor_core(fp, m, n, k, epi):
+    """int4 weights at 9-64 tokens, each weight expanded to bf16((q - z) s),
+    the prefill expansion, and accumulated in fp32: the tcgen05 decode path
+    from 17 tokens on, the CUDA-core GEMV below.  Cases: ragged row tiles,
+    tokens padded to 32 / 64, K / 128 = 8, 40, 32, 64, 9, 16, 86, 28, 2
+    groups (scale loads of 8 / 4 / 2 / 1 groups), row tiles shared by
+    several CTAs and CTAs covering whole tiles."""
+    w = synth.weight_bf16(50 + m, 0, 1, (n, k))
+    x = synth.uniform_bf16(51, m, (m, k), -2.0, 2.0)
+    r = synth.uniform_bf16(52, m, (m, n), -1.0, 1.0)
+    codes, scales, zeros = _quantized_on_device(fp, 2, w)
+    _, wd = quant.quantize_weight(w, 2)
+    # (q - z) s is exact in fp32 (at most 13 significant bits); one rounding to bf16
+    wb = quant.bf16_to_f32(synth.f32_to_bf16_bits(wd.astype(np.float32))).astype(np.float64)
+    xf = quant.bf16_to_f32(x).astype(np.float64)
+    nout = n // 2 if epi == 2 else n
+    out = empty(m * nout * (4 if epi == 3 else 2))
+    ws_b = fp.fp_op_linear_workspace_bytes(2, m, n, k)
+    ws = empty(max(ws_b, 16))
+    fp.fp_op_linear(2, epi, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(dev(r)), ptr(out),
+                    ptr(ws), ws_b)
+    if epi == 3:
+        got = host(out, np.float32).reshape(m, n).astype(np.float64)
+    else:
+        got = quant.bf16_to_f32(host(out, np.uint16)).reshape(m, nout).astype(np.float64)
+    # the tensor-core path multiplies the bf16 expansion; the CUDA-core GEMV
+    # removes the zero point in fp32 and so matches the exact dequantisation
+    tight = wb if m >= 17 else wd
+    for wm, tol in ((wd, TAU[2] / 4), (tight, 1e-4 if epi == 3 else 6e-3)):
+        y = xf @ wm.T
+        if epi == 1:
+            y = quant.bf16_to_f32(r).astype(np.float64) + y
+        elif epi == 2:
+            y = M.silu(y[:, :nout]) * y[:, nout:]
+        assert rel_err(got, y) <= tol, (m, n, k, epi, tol, rel_err(got, y))
+
+
 def test_linear_residual_in_place(fp):
     m, n, k = 5, 64, 256
     w = synth.weight_bf16(3, 0, 1, (n, k))
