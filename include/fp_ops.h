@@ -57,8 +57,10 @@ enum {
  * (codes / scales / zeros as fp_op_quantize writes them); fp32 accumulation.
  * Kernel choice depends on M, N and K: M <= 64 runs the decode GEMV (the
  * work is cut into equal ranges of (128-row block, K step), one per resident
- * CTA, and shared blocks are reduced from fp32 partials in a fixed order),
- * larger M the tcgen05 GEMM.  workspace: 16-byte aligned, at least
+ * CTA, and shared blocks are reduced from fp32 partials in a fixed order) --
+ * on the CUDA cores, except int4 with 17 <= M <= 64 and 16-byte aligned x and
+ * codes, which runs on tcgen05 with each weight expanded to bf16((q - z) s)
+ * as the prefill GEMM does -- larger M the tcgen05 GEMM.  workspace: 16-byte aligned, at least
  * fp_op_linear_workspace_bytes(wquant, M, N, K) bytes (may be NULL when that
  * is 0), else FP_ERR_INVALID_ARG.  Its leading bytes are ticket counters
  * that must be zero before the first call (e.g. a zeroed buffer); every call
