@@ -163,7 +163,9 @@ int fp_decode_step(fp_handle* h, const int32_t* host_in, int32_t* host_out);
  * (n graph replays, nothing crosses the host boundary; asynchronous). */
 int fp_decode_steps(fp_handle* h, int n);
 
-/* Kernel classes timed by fp_profile. */
+/* Kernel classes timed by fp_profile.  FP_K_EMBED is the embedding gather
+ * fused with the first block's pre-attention RMSNorm; FP_K_ARGMAX also moves
+ * every sequence's position past the pass. */
 enum {
   FP_K_EMBED = 0, FP_K_RMSNORM, FP_K_LIN_QKV, FP_K_ROPE_KV, FP_K_ATTN, FP_K_ATTN_COMBINE,
   FP_K_LIN_O, FP_K_LIN_GU, FP_K_LIN_DOWN, FP_K_LM_HEAD, FP_K_ARGMAX, FP_K_COUNT

@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       int g = (int)(begin % S);
       for (int q = 0; q < L; ++q, g = g + 1 == S ? 0 : g + 1) {
         const int s = q % XS;
-        if (q >= XS && (!mbar_wait(&xempty[s], ((q / XS) & 1) ^ 1) || *abort_flag)) {
+        if (q >= XS && (!mbar_wait_sleep(&xempty[s], ((q / XS) & 1) ^ 1) || *abort_flag)) {
           fail();
           break;
         }
@@ -210,8 +210,9 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       for (int q = 0; q < L; ++q, g = g + 1 == S ? 0 : g + 1) {
         const bool first = q == 0 || g == 0, last = g == S - 1 || q == L - 1;
         const int s = q % XS, a = q % NA;
-        if (first && seg > 0) ok = mbar_wait(&dempty, (seg - 1) & 1);  // the epilogue has read D
-        ok = ok && mbar_wait(&xfull[s], (q / XS) & 1) && mbar_wait(&afull[a], (q / NA) & 1) && !*abort_flag;
+        if (first && seg > 0) ok = mbar_wait_sleep(&dempty, (seg - 1) & 1);  // the epilogue has read D
+        ok = ok && mbar_wait_sleep(&xfull[s], (q / XS) & 1) && mbar_wait_sleep(&afull[a], (q / NA) & 1) &&
+             !*abort_flag;
         if (!ok) break;
         tc_fence_after();
         const uint64_t xd = sdesc(smem_u32(x_ring + s * G::kXBytes));
@@ -253,8 +254,10 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
     const uint32_t lane_base = tmem + ((uint32_t)(qd * 32) << 16);
     const long long row_bytes = (long long)S * 64;
 
-    // ---- this thread's code ring: its n-th own group (pair team + 2 n) in stage n % CS
-    uint8_t* my_ring = code_ring + (size_t)threadIdx.x * CK * 16;
+    // ---- this thread's code ring: its n-th own group (pair team + 2 n) in stage
+    // n % CS, chunk i at [stage][i][thread] (a warp's loads of one chunk are
+    // 512 contiguous bytes)
+    uint8_t* my_ring = code_ring + (size_t)threadIdx.x * 16;
     const int own = (L - team + 1) / 2;  // groups this team takes
     int ib = (int)((begin + team) / S), ig = (int)((begin + team) % S);  // (row tile, group) of the next copy
     const uint8_t* src = nullptr;
@@ -267,7 +270,7 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       if (n < own) {
         uint8_t* d = my_ring + (size_t)(n % CS) * G::kCodeBytes;
 #pragma unroll
-        for (int i = 0; i < CK; ++i) q4_cp16(d + i * 16, src + (long long)ig * 64 + i * 16);
+        for (int i = 0; i < CK; ++i) q4_cp16(d + i * (DW * 32 * 16), src + (long long)ig * 64 + i * 16);
         ig += 2;
         if (ig >= S) {
           while (ig >= S) ig -= S, ++ib;
@@ -317,7 +320,7 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
         uint4 wv[CK];
 #pragma unroll
         for (int i = 0; i < CK; ++i)
-          wv[i] = *reinterpret_cast<const uint4*>(my_ring + (size_t)(n % CS) * G::kCodeBytes + i * 16);
+          wv[i] = *reinterpret_cast<const uint4*>(my_ring + (size_t)(n % CS) * G::kCodeBytes + i * (DW * 32 * 16));
         issue(n + CS - 1);  // refills the stage read one own group ago
 
         const uint32_t sb = bf16_at(s_cur, j);

@@ -1,6 +1,7 @@
-// Row-wise kernels of the fingerprint block: embedding gather, RMSNorm,
-// RoPE + KV-cache append (with the int8 KV quantiser fused into the cache
-// write), greedy argmax and the position counter.
+// Row-wise kernels of the fingerprint block: embedding gather (alone or fused
+// with the first RMSNorm), RMSNorm, RoPE + KV-cache append (with the int8 KV
+// quantiser fused into the cache write) and greedy argmax (optionally
+// advancing the position counter).
 //
 // Components: embedding, normalisation and the LM head's greedy choice are
 // among the fingerprint's components (Sec. 1 "Our work"; Sec. 5.1); the KV
@@ -39,6 +40,63 @@ cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, in
                          cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
   return launch(embed_kernel, dim3(M), dim3(128), 0, s, tok, E, V, d, h, err);
+}
+
+// ------------------------------------------------------------------ embedding + RMSNorm
+// The embedding gather fused with the first block's pre-attention RMSNorm:
+// one CTA of 128 threads per token row writes h = E[tok] and
+// y = h * rsqrt(mean(h^2) + eps) * g (fp32 math), as embed_kernel followed
+// by rmsnorm_kernel would.  An out-of-range id gives h = y = 0 and err = 1.
+__global__ void embed_rmsnorm_kernel(const int32_t* __restrict__ tok, const uint16_t* __restrict__ E, int V, int d,
+                                     uint16_t* __restrict__ h, const uint16_t* __restrict__ g, float eps,
+                                     uint16_t* __restrict__ y, int32_t* err) {
+  pdl_trigger();
+  pdl_wait();
+  const long long m = blockIdx.x;
+  const int t = tok[m];
+  uint4* hr = reinterpret_cast<uint4*>(h + m * d);
+  uint4* yr = reinterpret_cast<uint4*>(y + m * d);
+  const int chunks = d / 8;
+  if (t < 0 || t >= V) {
+    if (threadIdx.x == 0 && err) atomicExch(err, 1);
+    for (int c = threadIdx.x; c < chunks; c += blockDim.x) hr[c] = yr[c] = make_uint4(0, 0, 0, 0);
+    return;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(E + (long long)t * d);
+  const uint4* gr = reinterpret_cast<const uint4*>(g);
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+    const uint4 v = ld_nc16(src + c);
+    hr[c] = v;
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = bf2x2f(w[i]);
+      ss += f.x * f.x + f.y * f.y;
+    }
+  }
+  ss = warp_sum(ss);
+  __shared__ float red[4];
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  const float inv = rsqrtf((red[0] + red[1] + red[2] + red[3]) / (float)d + eps);
+  for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+    const uint4 v = ld_nc16(src + c), gg = gr[c];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w}, gw[4] = {gg.x, gg.y, gg.z, gg.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = bf2x2f(w[i]), gf = bf2x2f(gw[i]);
+      o[i] = pack_bf2(f.x * inv * gf.x, f.y * inv * gf.y);
+    }
+    yr[c] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+cudaError_t launch_embed_rmsnorm(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h,
+                                 const uint16_t* g, float eps, uint16_t* y, int32_t* err, cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  return launch(embed_rmsnorm_kernel, dim3(M), dim3(128), 0, s, tok, E, V, d, h, g, eps, y, err);
 }
 
 // ------------------------------------------------------------------ RMSNorm
@@ -102,7 +160,7 @@ FP_DEV void better(float& bv, int& bi, float v, int i) {
 }
 
 __global__ void __cluster_dims__(kArgmaxCTAs, 1, 1) __launch_bounds__(256)
-    argmax_kernel(const float* __restrict__ logits, int V, int32_t* __restrict__ out) {
+    argmax_kernel(const float* __restrict__ logits, int V, int32_t* __restrict__ out, int32_t* pos, int by) {
   __shared__ float sv[8];
   __shared__ int si[8];
   __shared__ float cv;
@@ -158,13 +216,14 @@ __global__ void __cluster_dims__(kArgmaxCTAs, 1, 1) __launch_bounds__(256)
       better(b, i, *rv, *ri);
     }
     out[row] = i == 0x7fffffff ? 0 : i;
+    if (pos) pos[row] += by;  // the sequence's next position (the decode step is complete)
   }
   cluster.sync();  // keep the winners alive until CTA 0 has read them
 }
 
-cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s) {
+cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s, int32_t* pos, int by) {
   if (M <= 0) return cudaSuccess;
-  return launch(argmax_kernel, dim3(kArgmaxCTAs, M), dim3(256), 0, s, logits, V, out);
+  return launch(argmax_kernel, dim3(kArgmaxCTAs, M), dim3(256), 0, s, logits, V, out, pos, by);
 }
 
 // ------------------------------------------------------------------ RoPE + KV append
@@ -261,18 +320,6 @@ cudaError_t launch_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_he
       return launch(rope_kv_kernel<128, FP_KV_INT8>, dim3(blocks), dim3(256), 0, s, qkv, B, S, row_stride, n_heads, kv, pos, rope_cs, err);
   }
   return cudaGetLastError();
-}
-
-// ------------------------------------------------------------------ positions
-__global__ void advance_kernel(int32_t* pos, int B, int by) {
-  pdl_trigger();
-  pdl_wait();
-  int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < B) pos[b] += by;
-}
-
-cudaError_t launch_advance(int32_t* pos, int B, int by, cudaStream_t s) {
-  return launch(advance_kernel, dim3((B + 127) / 128), dim3(128), 0, s, pos, B, by);
 }
 
 }  // namespace fpk

@@ -284,12 +284,14 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
     ~PdlScope() { g_pdl = false; }
   } pdl_scope;
   h->tr.start();
-  LTRY(launch_embed(tok, M, h->embed, a.vocab, d, h->h, h->err, s), FP_K_EMBED);
+  // the embedding and the first block's pre-attention RMSNorm in one kernel
+  LTRY(launch_embed_rmsnorm(tok, M, h->embed, a.vocab, d, h->h, h->L[0].attn_norm, a.rms_eps, h->y, h->err, s),
+       FP_K_EMBED);
   h->tr.boundary();
   for (int l = 0; l < a.n_layers; ++l) {
     Layer& Ly = h->L[l];
     const fp_kv_view kv = h->kv(l);
-    LTRY(launch_rmsnorm(h->h, M, d, 1, 0, Ly.attn_norm, a.rms_eps, h->y, s), FP_K_RMSNORM);
+    if (l > 0) LTRY(launch_rmsnorm(h->h, M, d, 1, 0, Ly.attn_norm, a.rms_eps, h->y, s), FP_K_RMSNORM);
     const Mat& Q = Ly.mat[FP_M_QKV];
     LTRY(launch_linear(h->wq, FP_EPI_STORE, h->y, M, Q.N, Q.K, Q.codes, Q.scales, Q.zeros, nullptr, h->qkv,
                        h->lin_ws, h->lin_ws_bytes, s, h->err),
@@ -330,8 +332,8 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
   LTRY(launch_linear(FP_W_BF16, FP_EPI_F32, h->ylast, B, a.vocab, d, h->lm_head, nullptr, nullptr, nullptr,
                      h->logits, h->lin_ws, h->lin_ws_bytes, s, h->err),
        FP_K_LM_HEAD);
-  LTRY(launch_argmax(h->logits, B, a.vocab, h->tokens, s), FP_K_ARGMAX);
-  LTRY(launch_advance(h->pos, B, S, s), FP_K_ARGMAX);
+  // the greedy token, and each sequence's position moves past this pass
+  LTRY(launch_argmax(h->logits, B, a.vocab, h->tokens, s, h->pos, S), FP_K_ARGMAX);
   h->tr.boundary();
   h->last_rows = M;
   return FP_OK;

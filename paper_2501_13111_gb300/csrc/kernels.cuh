@@ -22,10 +22,13 @@ cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, in
                          int32_t* err, cudaStream_t s);
 cudaError_t launch_rmsnorm(const uint16_t* x, int M, int d, int row_stride, int row_offset,
                            const uint16_t* g, float eps, uint16_t* y, cudaStream_t s);
-cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s);
+// pos (optional): pos[row] += by once row's token is written.
+cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaStream_t s, int32_t* pos = nullptr,
+                          int by = 0);
+cudaError_t launch_embed_rmsnorm(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h,
+                                 const uint16_t* g, float eps, uint16_t* y, int32_t* err, cudaStream_t s);
 cudaError_t launch_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_heads, const fp_kv_view& kv,
                            const int32_t* pos, const float* rope_cs, int32_t* err, cudaStream_t s);
-cudaError_t launch_advance(int32_t* pos, int B, int by, cudaStream_t s);
 
 // ---- attention (fp_attention.cu)
 size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len);
