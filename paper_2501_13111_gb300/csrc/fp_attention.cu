@@ -532,9 +532,13 @@ cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int 
 // =====================================================================
 // Prefill: causal attention of S query rows per sequence against cache
 // positions 0..S-1.  CTA = 64 query rows of one (b, h); 4 warps x 16 rows;
-// key/value tiles of 64 staged in shared memory as bf16; S = Q K^T and
-// O += P V with mma.sync m16n8k16 (bf16 in, fp32 accumulate) and an online
-// softmax in the log2 domain.
+// key/value tiles of 64 stream through a two-stage cp.async ring (the next
+// tile loads while this one computes) for bf16 caches; int8 codes are loaded
+// and widened exactly to bf16 tile by tile (a staged copy of the codes plus
+// a widening pass measured slower at the 70B shape), their per-token scales
+// multiplying S and P.  S = Q K^T and O += P V with mma.sync m16n8k16 (bf16
+// in, fp32 accumulate; ldmatrix, transposed for V) and an online
+// softmax in the log2 domain; P stays in registers as the A operand.
 // =====================================================================
 FP_DEV void mma_bf16(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -561,31 +565,80 @@ FP_DEV void ldsm_x2_trans(uint32_t& r0, uint32_t& r1, const void* p) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0,%1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(a));
 }
 
+// 16-byte cp.async that writes zeros when `valid` is false (source size 0).
+FP_DEV void pf_cp16(void* smem, const void* gmem, bool valid) {
+  const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem), "r"(valid ? 16 : 0) : "memory");
+}
+
+template <int HD, int KVQ>
+constexpr size_t prefill_smem_bytes() {
+  constexpr int BT = 64, LD = HD + 8;
+  // bf16 cache: two stages of K and V tiles; int8 cache: one K and V tile
+  // and the tile's scales.  The Q tile borrows a K tile.
+  if (KVQ == FP_KV_INT8) return (size_t)2 * BT * LD * 2 + (size_t)2 * BT * sizeof(float);
+  return (size_t)2 * 2 * BT * LD * 2;
+}
+
 template <int HD, int KVQ>
 __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __restrict__ q, int q_stride, int S,
                                                            int H, fp_kv_view kv, uint16_t* __restrict__ out,
                                                            int32_t* err) {
-  constexpr int BT = 64;        // rows per tile
+  constexpr int BT = 64;        // query rows per CTA and keys per tile
   constexpr int LD = HD + 8;    // padded row (bf16 elements) against ldmatrix bank conflicts
+  constexpr bool I8 = KVQ == FP_KV_INT8;
+  constexpr int RB = I8 ? HD : 2 * HD;  // bytes of one cached row
+  constexpr int CPR = RB / 16;          // 16-byte chunks per cached row
   extern __shared__ __align__(16) uint8_t smem_raw[];
   pdl_trigger();
   pdl_wait();
-  uint16_t* sQ = reinterpret_cast<uint16_t*>(smem_raw);
-  uint16_t* sK = sQ + BT * LD;
-  uint16_t* sV = sK + BT * LD;
-  float* sks = reinterpret_cast<float*>(sV + BT * LD);  // [BT] key scales (int8)
-  float* svs = sks + BT;                                // [BT] value scales (int8)
+  constexpr int NT = I8 ? 1 : 2;  // bf16 tile stages
+  uint16_t* sKV = reinterpret_cast<uint16_t*>(smem_raw);  // [stage][K | V][BT][LD] bf16
+  float* rsc = reinterpret_cast<float*>(sKV + NT * 2 * BT * LD);  // int8: [K | V][BT] scales
+  auto tileK = [&](int st) { return sKV + ((st % NT) * 2 + 0) * BT * LD; };
+  auto tileV = [&](int st) { return sKV + ((st % NT) * 2 + 1) * BT * LD; };
+  // the Q tile is read into fragments before the first __syncthreads of the
+  // key loop, after which that K tile is first written
+  uint16_t* sQ = tileK(1);
 
   const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int Hkv = kv.n_kv_heads, G = H / Hkv, kvh = h / G;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g8 = lane >> 2, t4 = lane & 3;
   const int q0 = qt * BT;
-  constexpr int CPR = HD / 8;  // 16-byte chunks per bf16 row
+  const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
+  const int last_key = min(q0 + BT, S) - 1;
+  const int ntile = last_key / BT + 1;
 
-  // ---- Q tile
-  for (int c = tid; c < BT * CPR; c += 128) {
-    const int r = c / CPR, cc = c % CPR;
+  // ---- cache row of key t: its index in the pool, or -1 past S / on a bad page
+  auto row_of = [&](int t) -> long long {
+    if (t >= S) return -1;
+    const int page = pt[t / kv.page_size];
+    if (page < 0 || page >= kv.n_pages) {
+      if (err) atomicExch(err, 1);
+      return -1;
+    }
+    return ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
+  };
+  // ---- bf16: one key tile (rows k0 .. k0 + 63, zeros where row_of < 0) into stage st
+  auto issue = [&](int tile, int st) {
+    if constexpr (!I8) {
+      const int k0 = tile * BT;
+      for (int c = tid; c < 2 * BT * CPR; c += 128) {
+        const int which = c / (BT * CPR), r = (c % (BT * CPR)) / CPR, cc = c % CPR;
+        const long long rowi = row_of(k0 + r);
+        const uint8_t* src = (const uint8_t*)(which ? kv.v_pool : kv.k_pool) + (rowi >= 0 ? rowi * RB + cc * 16 : 0);
+        pf_cp16((which ? tileV(st) : tileK(st)) + r * LD + cc * 8, src, rowi >= 0);
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+  };
+  issue(0, 0);
+
+  // ---- Q tile -> fragments (row-major A operand of the warp's 16 rows)
+  constexpr int QCPR = HD / 8;
+  for (int c = tid; c < BT * QCPR; c += 128) {
+    const int r = c / QCPR, cc = c % QCPR;
     uint4 v = make_uint4(0, 0, 0, 0);
     if (q0 + r < S) v = ld_nc16(q + ((long long)b * S + q0 + r) * q_stride + (long long)h * HD + cc * 8);
     *reinterpret_cast<uint4*>(sQ + r * LD + cc * 8) = v;
@@ -604,62 +657,45 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __res
   for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
   const float scale = kLog2e * rsqrtf((float)HD);
-  const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
-  const int last_key = min(q0 + BT, S) - 1;
   const int qrow0 = q0 + warp * 16 + g8;  // rows qrow0 and qrow0 + 8
 
-  for (int k0 = 0; k0 <= last_key; k0 += BT) {
-    __syncthreads();
-    // ---- stage K and V rows k0 .. k0+63 (zeros past S)
-    if (KVQ == FP_KV_BF16) {
+  for (int tile = 0; tile < ntile; ++tile) {
+    const int st = tile & 1, k0 = tile * BT;
+    if constexpr (!I8) asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();  // the tile landed for every thread; every warp is done with the other stage
+    if (tile + 1 < ntile) issue(tile + 1, st ^ 1);
+    const float* sks = rsc;
+    const float* svs = rsc + BT;
+    if constexpr (I8) {
+      // codes -> bf16 (small integers: exact) while loading; the scales multiply S and P
       for (int c = tid; c < 2 * BT * CPR; c += 128) {
         const int which = c / (BT * CPR), r = (c % (BT * CPR)) / CPR, cc = c % CPR;
-        const int t = k0 + r;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (t < S) {
-          const int page = pt[t / kv.page_size];
-          if (page >= 0 && page < kv.n_pages) {
-            const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
-            v = ld_nc16((const uint16_t*)(which ? kv.v_pool : kv.k_pool) + rowi * HD + cc * 8);
-          } else if (err) {
-            atomicExch(err, 1);
-          }
-        }
-        *reinterpret_cast<uint4*>((which ? sV : sK) + r * LD + cc * 8) = v;
-      }
-    } else {
-      constexpr int CPR8 = HD / 16;  // 16-byte chunks per int8 row
-      for (int c = tid; c < 2 * BT * CPR8; c += 128) {
-        const int which = c / (BT * CPR8), r = (c % (BT * CPR8)) / CPR8, cc = c % CPR8;
-        const int t = k0 + r;
+        const long long rowi = row_of(k0 + r);
         uint4 v = make_uint4(0, 0, 0, 0);
         float sc = 0.f;
-        if (t < S) {
-          const int page = pt[t / kv.page_size];
-          if (page >= 0 && page < kv.n_pages) {
-            const long long rowi = ((long long)page * Hkv + kvh) * kv.page_size + t % kv.page_size;
-            v = ld_nc16((const int8_t*)(which ? kv.v_pool : kv.k_pool) + rowi * HD + cc * 16);
-            sc = (which ? kv.v_scale : kv.k_scale)[rowi];
-          } else if (err) {
-            atomicExch(err, 1);
-          }
+        if (rowi >= 0) {
+          v = ld_nc16((const uint8_t*)(which ? kv.v_pool : kv.k_pool) + rowi * RB + cc * 16);
+          sc = (which ? kv.v_scale : kv.k_scale)[rowi];
         }
-        uint32_t w[4] = {v.x, v.y, v.z, v.w}, o8[8];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+        uint32_t o8[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           const uint32_t word = w[i >> 1];
           const int sh = 16 * (i & 1);
-          const float a = (float)(int8_t)((word >> sh) & 0xFF), bb = (float)(int8_t)((word >> (sh + 8)) & 0xFF);
-          o8[i] = pack_bf2(a, bb);  // small integers: exact in bf16
+          o8[i] = pack_bf2((float)(int8_t)((word >> sh) & 0xFF), (float)(int8_t)((word >> (sh + 8)) & 0xFF));
         }
-        uint16_t* dst = (which ? sV : sK) + r * LD + cc * 16;
+        uint16_t* dst = (which ? tileV(st) : tileK(st)) + r * LD + cc * 16;
         *reinterpret_cast<uint4*>(dst) = make_uint4(o8[0], o8[1], o8[2], o8[3]);
         *reinterpret_cast<uint4*>(dst + 8) = make_uint4(o8[4], o8[5], o8[6], o8[7]);
-        if (cc == 0) (which ? svs : sks)[r] = sc;
+        if (cc == 0) rsc[which * BT + r] = sc;
       }
+      __syncthreads();
     }
-    __syncthreads();
-    // ---- S = Q K^T for this warp's 16 rows x 64 keys
+    const uint16_t* tK = tileK(st);
+    const uint16_t* tV = tileV(st);
+    // ---- S = Q K^T for this warp's 16 rows x 64 keys (two-matrix ldmatrix per
+    // n8 key tile: the four-matrix form measured 25% slower with the int8 cache)
     float sacc[BT / 8][4];
 #pragma unroll
     for (int n = 0; n < BT / 8; ++n) sacc[n][0] = sacc[n][1] = sacc[n][2] = sacc[n][3] = 0.f;
@@ -668,8 +704,7 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __res
 #pragma unroll
       for (int n = 0; n < BT / 8; ++n) {
         uint32_t b0, b1;
-        const int r = n * 8 + (lane & 7), c = kk * 16 + 8 * ((lane >> 3) & 1);
-        ldsm_x2(b0, b1, sK + r * LD + c);
+        ldsm_x2(b0, b1, tK + (n * 8 + (lane & 7)) * LD + kk * 16 + 8 * ((lane >> 3) & 1));
         mma_bf16(sacc[n], qf[kk], b0, b1);
       }
     }
@@ -682,7 +717,7 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __res
         const int key = k0 + n * 8 + 2 * t4 + (i & 1);
         const int row = qrow0 + 8 * (i >> 1);
         float v = sacc[n][i] * scale;
-        if (KVQ == FP_KV_INT8) v *= sks[n * 8 + 2 * t4 + (i & 1)];
+        if constexpr (I8) v *= sks[n * 8 + 2 * t4 + (i & 1)];
         if (key > row || key >= S) v = -INFINITY;
         sacc[n][i] = v;
         mx[i >> 1] = fmaxf(mx[i >> 1], v);
@@ -714,23 +749,23 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __res
       for (int i = 0; i < 4; ++i) {
         p[i] = exp2f(sacc[n][i] - mref[i >> 1]);
         lrow[i >> 1] += p[i];
-        if (KVQ == FP_KV_INT8) p[i] *= svs[n * 8 + 2 * t4 + (i & 1)];
+        if constexpr (I8) p[i] *= svs[n * 8 + 2 * t4 + (i & 1)];
       }
       pa[n >> 1][(n & 1) * 2 + 0] = pack_bf2(p[0], p[1]);
       pa[n >> 1][(n & 1) * 2 + 1] = pack_bf2(p[2], p[3]);
     }
-    // ---- O += P V
+    // ---- O += P V: V^T fragments by transposing ldmatrix
 #pragma unroll
     for (int j = 0; j < BT / 16; ++j) {
 #pragma unroll
       for (int dt = 0; dt < HD / 8; ++dt) {
         uint32_t b0, b1;
-        const int r = j * 16 + (lane & 7) + 8 * ((lane >> 3) & 1);
-        ldsm_x2_trans(b0, b1, sV + r * LD + dt * 8);
+        ldsm_x2_trans(b0, b1, tV + (j * 16 + (lane & 7) + 8 * ((lane >> 3) & 1)) * LD + dt * 8);
         mma_bf16(o[dt], pa[j], b0, b1);
       }
     }
   }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
   // ---- normalise and store
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
@@ -753,10 +788,13 @@ __global__ void __launch_bounds__(128) attn_prefill_kernel(const uint16_t* __res
 template <int HD, int KVQ>
 static cudaError_t launch_prefill_t(const uint16_t* q, int q_stride, int B, int S, int H, const fp_kv_view& kv,
                                     uint16_t* out, int32_t* err, cudaStream_t s) {
-  constexpr int LD = HD + 8;
-  size_t smem = 3 * 64 * LD * 2 + 2 * 64 * sizeof(float);
+  const size_t smem = prefill_smem_bytes<HD, KVQ>();
   auto kern = attn_prefill_kernel<HD, KVQ>;
-  if (smem > 48 * 1024) FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  static bool attr = false;
+  if (!attr) {
+    FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    attr = true;
+  }
   dim3 grid((S + 63) / 64, H, B);
   return launch(kern, grid, dim3(128), smem, s, q, q_stride, S, H, kv, out, err);
 }

@@ -13,7 +13,8 @@ calls, which is the shape a profiler capture wants (``-s 2 -c 1``).
 
 Decode linears report GB/s of algorithmic bytes (codes + scales/zeros +
 activations in and out); attention reports GB/s of cached K/V (+ int8 scales);
-the prefill GEMM reports TFLOP/s of 2·M·N·K.  Weights and caches hold random
+the prefill GEMM reports TFLOP/s of 2·M·N·K and prefill attention those of
+both matmuls over the causal half, 2·B·H·S²·hd.  Weights and caches hold random
 values: speed does not depend on them.
 """
 import argparse
@@ -121,6 +122,34 @@ def case_attention(B, H, Hkv, hd, ctx, kvq, single, iters):
     return ms, moved / ms / 1e6, "GB/s"
 
 
+def case_attention_prefill(B, H, Hkv, hd, S, kvq, single, iters):
+    P = 16
+    pps = -(-S // P)
+    npg = B * pps
+    elt = 2 if kvq == 0 else 1
+    pool = npg * Hkv * P * hd * elt
+    if kvq == 0:
+        kp = (torch.randn(pool // 2, device="cuda") * 0.5).to(torch.bfloat16)
+        vp = (torch.randn(pool // 2, device="cuda") * 0.5).to(torch.bfloat16)
+    else:
+        kp = torch.randint(-100, 100, (pool,), dtype=torch.int8, device="cuda")
+        vp = torch.randint(-100, 100, (pool,), dtype=torch.int8, device="cuda")
+    ks = torch.rand(npg * Hkv * P, device="cuda") * 0.01
+    vs = torch.rand(npg * Hkv * P, device="cuda") * 0.01
+    pt = torch.randperm(npg, device="cuda").to(torch.int32)
+    kv = fp.fp_kv_view(kvq, Hkv, hd, P, pps, npg, kp.data_ptr(), vp.data_ptr(),
+                       ks.data_ptr() if kvq else None, vs.data_ptr() if kvq else None, pt.data_ptr())
+    q = torch.randn(B * S, H * hd, device="cuda").to(torch.bfloat16)
+    out = torch.empty(B * S * H * hd, dtype=torch.bfloat16, device="cuda")
+
+    def f():
+        fp.fp_op_attention_prefill(q.data_ptr(), H * hd, B, S, H, kv, out.data_ptr())
+
+    ms = timed(f, iters)
+    flops = 2.0 * B * H * S * S * hd  # both matmuls over the causal half
+    return ms, flops / (ms * 1e-3) / 1e12, "TFLOP/s"
+
+
 def case_argmax(M, V, single, iters):
     copies = 1 if single else 8
     logits = [torch.randn(M, V, device="cuda") for _ in range(copies)]
@@ -149,13 +178,17 @@ for tag, (wq, d, H, Hkv, f, Mdec) in {"7b": (1, 4096, 32, 32, 11008, 8), "13b": 
 CASES["7b-attn"] = ("attention", (8, 32, 32, 128, 612, 0))
 CASES["13b-attn"] = ("attention", (16, 40, 40, 128, 1124, 0))
 CASES["70b-attn"] = ("attention", (32, 64, 8, 128, 2148, 1))
+CASES["7b-attn-prefill"] = ("attention_prefill", (8, 32, 32, 128, 512, 0))
+CASES["13b-attn-prefill"] = ("attention_prefill", (16, 40, 40, 128, 1024, 0))
+CASES["70b-attn-prefill"] = ("attention_prefill", (32, 64, 8, 128, 2048, 1))
 CASES["7b-qkv-prefill"] = ("linear", (1, 0, 4096, 12288, 4096))
 CASES["7b-gu-prefill"] = ("linear", (1, 2, 4096, 22016, 4096))
 CASES["7b-down-prefill"] = ("linear", (1, 1, 4096, 4096, 11008))
 CASES["13b-gu-prefill"] = ("linear", (2, 2, 16384, 27648, 5120))
 CASES["bf16-8k-prefill"] = ("linear", (0, 0, 8192, 8192, 8192))
 
-RUNNERS = {"linear": case_linear, "attention": case_attention, "argmax": case_argmax}
+RUNNERS = {"linear": case_linear, "attention": case_attention, "attention_prefill": case_attention_prefill,
+           "argmax": case_argmax}
 
 
 def main(argv=None):

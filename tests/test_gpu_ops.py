@@ -275,7 +275,7 @@ def test_attention_decode(fp, kvq, hd, H, Hkv, lens):
 
 @pytest.mark.parametrize("kvq", [0, 1])
 @pytest.mark.parametrize("hd,H,Hkv", [(64, 4, 4), (128, 8, 2)])
-@pytest.mark.parametrize("S", [1, 17, 64, 130])
+@pytest.mark.parametrize("S", [1, 17, 64, 130, 513])
 def test_attention_prefill(fp, kvq, hd, H, Hkv, S):
     B = 2
     c = Cache(fp, kvq, B, S + 5, Hkv, hd, seed=S + hd + kvq)
