@@ -802,6 +802,8 @@ static cudaError_t launch_prefill_t(const uint16_t* q, int q_stride, int B, int 
 cudaError_t launch_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
                                      const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s) {
   if (B <= 0 || S <= 0) return cudaSuccess;
+  if (attention_prefill_tc_ok(B, S, n_heads, kv, q, q_stride))
+    return launch_attention_prefill_tc(q, q_stride, B, S, n_heads, kv, out, err, s);
   if (kv.head_dim == 64)
     return kv.kvquant == FP_KV_BF16 ? launch_prefill_t<64, FP_KV_BF16>(q, q_stride, B, S, n_heads, kv, out, err, s)
                                     : launch_prefill_t<64, FP_KV_INT8>(q, q_stride, B, S, n_heads, kv, out, err, s);

@@ -37,6 +37,10 @@ int attention_decode_launches(int B, int n_kv_heads, int max_len);
 cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, const fp_kv_view& kv,
                                     const int32_t* len, int len_add, int max_len, uint16_t* out, void* ws,
                                     int32_t* err, cudaStream_t s, cudaError_t* second = nullptr);
+// tcgen05 prefill attention (bf16 cache, head_dim 128, 16-token pages; fp_attn_tc.cu)
+bool attention_prefill_tc_ok(int B, int S, int n_heads, const fp_kv_view& kv, const void* q, int q_stride);
+cudaError_t launch_attention_prefill_tc(const uint16_t* q, int q_stride, int B, int S, int n_heads,
+                                        const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s);
 cudaError_t launch_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
                                      const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s);
 
