@@ -3,24 +3,28 @@
 //
 // o = softmax(q K^T / sqrt(hd) + causal mask) V for the S query rows of one
 // (sequence, head) against cache positions 0..S-1 (Sec. 5.1: the block's
-// attention).  CTA = 128 query rows of one (b, h), key tiles of 128:
+// attention).  CTA = 128 query rows of one (b, h), key tiles of 128; two
+// CTAs per SM (256 TMEM columns and 97 KiB of shared memory each), so one
+// CTA's softmax overlaps the other's MMAs and loads:
 //   warp 0      TMA: the Q tile once (two 64-column boxes of the q rows), then
-//               each key tile's K and V rows page by page (a [16][64] box per
-//               16-token page and half of head_dim, 128-byte swizzle) into a
-//               two-stage ring (kvfull / kvempty);
-//   warp 1      allocates 512 TMEM columns and issues the MMAs: S = Q K^T
-//               (M 128 queries, N 128 keys, K 16 over head_dim; K-major
-//               operands) into one of two score buffers, then O += P V
-//               (A = P from TMEM, B = V read MN-major from the same tile);
-//   warps 2-5   softmax, one query row (TMEM lane) per thread: the row's 128
-//               scores (tcgen05.ld), scale and causal mask, running maximum in
-//               the log2 domain, P = 2^(s - m) as bf16 into TMEM, the O rescale
-//               when the maximum grows, and at the end o / l stored as bf16.
-// TMEM columns: scores S0 [0, 128), S1 [128, 256), O [256, 384), P [384, 448).
-// The scores of key tile t + 1 are computed while the softmax works on tile
-// t.  Every mbarrier wait is bounded (error 2 past the limit); a page id out
-// of range reads zeros and sets error 1.
+//               per key tile its K rows and its V rows page by page (a
+//               [16][64] box per 16-token page and half of head_dim, 128-byte
+//               swizzle); K(t + 1) loads once S(t) has read K(t), V(t + 1)
+//               once P(t) V(t) has read V(t);
+//   warp 1      allocates the TMEM and issues the MMAs: S = Q K^T (M 128
+//               queries, N 128 keys, K 16 over head_dim; K-major operands),
+//               then O += P V (A = P from TMEM, B = V read MN-major);
+//   warps 2-5   softmax, one query row (TMEM lane) per thread, over 32-column
+//               chunks: a first pass for the row maximum (log2 domain), a
+//               second for P = 2^(s - m) written as bf16 over the scores
+//               already read.  The reference maximum m only moves when a tile
+//               raises it by more than 2^8 (O and the row sum are rescaled
+//               then); P never exceeds 256, and o / l is exact either way.
+// TMEM columns: scores S [0, 128) with P over [0, 64), O [128, 256).  Every
+// mbarrier wait is bounded (error 2 past the limit); a page id out of range
+// reads zeros and sets error 1.
 #include <algorithm>
+#include <type_traits>
 
 #include "common.cuh"
 #include "kernels.cuh"
@@ -31,12 +35,13 @@ namespace fpk {
 constexpr int kPaB = 128;  // query rows per CTA = keys per tile
 constexpr int kPaHD = 128;
 constexpr int kPaThreads = 192;
-constexpr uint32_t kPaTmemCols = 512;
-constexpr uint32_t kPaS0 = 0, kPaO = 256, kPaP = 384;
+constexpr uint32_t kPaTmemCols = 256;
+constexpr uint32_t kPaS = 0, kPaO = 128;
 constexpr int kPaHalf = kPaB * 128;          // bytes of one [128 rows][64 bf16] swizzled half
 constexpr int kPaTile = 2 * kPaHalf;         // one [128][128] bf16 operand
-constexpr int kPaSmem = kPaTile + 2 * 2 * kPaTile + 1024;  // Q, two stages of K and V, alignment
+constexpr int kPaSmem = 3 * kPaTile + 1024;  // Q, K, V, alignment
 constexpr float kPaLog2e = 1.4426950408889634f;
+constexpr float kPaSlack = 8.f;  // log2 of the largest P allowed before the reference maximum moves
 
 // Shared-memory descriptor of an MN-major operand with 128-byte swizzle:
 // 64-element atoms along MN `lbo` bytes apart, 8-row groups along K 1024
@@ -51,20 +56,38 @@ FP_DEV uint64_t sdesc_mn(uint32_t saddr, uint32_t lbo) {
   return d;
 }
 
-__global__ void __launch_bounds__(kPaThreads, 1)
+// 16 consecutive 32-bit columns into this thread's TMEM lane.
+FP_DEV void pa_st16(uint32_t taddr, const uint32_t* r) { tc_st16(taddr, r); }
+
+// 2^x by the hardware approximation (subnormal results flush to zero: P
+// values below 2^-126 carry no weight next to the row's maximum of 1 .. 256).
+FP_DEV float pa_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// (lo, hi) -> bf16x2, round to nearest even.
+FP_DEV uint32_t pa_pack(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+__global__ void __launch_bounds__(kPaThreads, 2)
     attn_prefill_tc_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                            const __grid_constant__ CUtensorMap map_v, int S, int H, int Hkv, int page_size,
                            const int32_t* __restrict__ page_table, int pages_per_seq, int n_pages,
                            uint16_t* __restrict__ out, int32_t* err) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t qfull, kvfull[2], kvempty[2], sfull[2], sempty[2], pfull, ofull, mma_done;
+  __shared__ uint64_t qfull, kfull, kempty, vfull, vempty, sfull, pfull, ofull, mma_done;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_word;
   volatile int* abort_flag = &abort_word;
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sQ = smem;
-  auto sK = [&](int st) { return smem + kPaTile + st * 2 * kPaTile; };
-  auto sV = [&](int st) { return smem + kPaTile + st * 2 * kPaTile + kPaTile; };
+  uint8_t* sK = smem + kPaTile;
+  uint8_t* sV = smem + 2 * kPaTile;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int kvh = h / (H / Hkv);
@@ -78,12 +101,11 @@ __global__ void __launch_bounds__(kPaThreads, 1)
   pdl_trigger();
   if (threadIdx.x == 0) {
     mbar_init(&qfull, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&kvfull[i], 1);
-      mbar_init(&kvempty[i], 1);
-      mbar_init(&sfull[i], 1);
-      mbar_init(&sempty[i], 4);
-    }
+    mbar_init(&kfull, 1);
+    mbar_init(&kempty, 1);
+    mbar_init(&vfull, 1);
+    mbar_init(&vempty, 1);
+    mbar_init(&sfull, 1);
     mbar_init(&pfull, 4);
     mbar_init(&ofull, 1);
     mbar_init(&mma_done, 1);
@@ -105,73 +127,79 @@ __global__ void __launch_bounds__(kPaThreads, 1)
   if (warp == 0) {
     // ---------------- TMA producer
     if (lane == 0) {
+      const int32_t* pt = page_table + (long long)b * pages_per_seq;
+      // the key tile's rows, page by page (rows past S, or of a bad page, read zeros)
+      auto load_rows = [&](const CUtensorMap* map, uint8_t* dst, int t, uint64_t* bar) {
+        int rows[kPaB / 16];  // the page ids are all read before the first copy is issued
+#pragma unroll
+        for (int pg = 0; pg < kPaB / 16; ++pg) {
+          const int key0 = t * kPaB + pg * 16;
+          rows[pg] = key0 < S ? __ldg(pt + key0 / page_size) : -1;
+        }
+#pragma unroll
+        for (int pg = 0; pg < kPaB / 16; ++pg) {
+          int row = -16;
+          if (t * kPaB + pg * 16 < S) {
+            if (rows[pg] >= 0 && rows[pg] < n_pages) row = (rows[pg] * Hkv + kvh) * page_size;
+            else if (err) atomicExch(err, 1);
+          }
+          tma_load_2d(dst + pg * 2048, map, 0, row, bar);
+          tma_load_2d(dst + kPaHalf + pg * 2048, map, 64, row, bar);
+        }
+      };
       mbar_expect_tx(&qfull, kPaTile);
       tma_load_2d(sQ, &map_q, h * kPaHD, b * S + q0, &qfull);
       tma_load_2d(sQ + kPaHalf, &map_q, h * kPaHD + 64, b * S + q0, &qfull);
-      const int32_t* pt = page_table + (long long)b * pages_per_seq;
-      int issued = 0;
+      int kiss = 0, viss = 0;
       for (int t = 0; t < nt; ++t) {
-        const int st = t & 1;
-        if (t >= 2 && (!mbar_wait(&kvempty[st], ((t >> 1) & 1) ^ 1) || *abort_flag)) {
+        if (t > 0 && (!mbar_wait_sleep(&kempty, (t - 1) & 1) || *abort_flag)) {
           fail();
           break;
         }
-        mbar_expect_tx(&kvfull[st], 2 * kPaTile);
-        for (int pg = 0; pg < kPaB / 16; ++pg) {
-          const int key0 = t * kPaB + pg * 16;
-          int row = -16;  // wholly outside the pool: the box reads zeros
-          if (key0 < S) {
-            const int page = pt[key0 / page_size];
-            if (page >= 0 && page < n_pages) row = (page * Hkv + kvh) * page_size;
-            else if (err) atomicExch(err, 1);
-          }
-#pragma unroll
-          for (int half = 0; half < 2; ++half) {
-            tma_load_2d(sK(st) + half * kPaHalf + pg * 2048, &map_k, half * 64, row, &kvfull[st]);
-            tma_load_2d(sV(st) + half * kPaHalf + pg * 2048, &map_v, half * 64, row, &kvfull[st]);
-          }
+        mbar_expect_tx(&kfull, kPaTile);
+        load_rows(&map_k, sK, t, &kfull);
+        kiss = t + 1;
+        if (t > 0 && (!mbar_wait_sleep(&vempty, (t - 1) & 1) || *abort_flag)) {
+          fail();
+          break;
         }
-        issued = t + 1;
+        mbar_expect_tx(&vfull, kPaTile);
+        load_rows(&map_v, sV, t, &vfull);
+        viss = t + 1;
       }
       // copies still in flight land before the CTA leaves
       mbar_wait(&qfull, 0);
-      for (int j = max(0, issued - 2); j < issued; ++j) mbar_wait(&kvfull[j & 1], (j >> 1) & 1);
+      if (kiss > 0) mbar_wait(&kfull, (kiss - 1) & 1);
+      if (viss > 0) mbar_wait(&vfull, (viss - 1) & 1);
     }
   } else if (warp == 1) {
     // ---------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_s = tc_idesc(kPaB, kPaB);             // Q, K both K-major
+      constexpr uint32_t idesc_s = tc_idesc(kPaB, kPaB);                // Q, K both K-major
       constexpr uint32_t idesc_o = tc_idesc(kPaB, kPaHD) | (1u << 16);  // V MN-major
-      bool ok = mbar_wait(&qfull, 0);
-      auto issue_s = [&](int t) -> bool {
-        const int st = t & 1, sb = t & 1;
-        if (!mbar_wait(&kvfull[st], (t >> 1) & 1)) return false;
-        if (t >= 2 && !mbar_wait(&sempty[sb], ((t >> 1) & 1) ^ 1)) return false;
+      bool ok = mbar_wait_sleep(&qfull, 0);
+      const uint32_t q = smem_u32(sQ), k = smem_u32(sK), v = smem_u32(sV);
+      for (int t = 0; t < nt && ok; ++t) {
+        // S(t) overwrites P(t - 1): its P V has completed (in order with this thread's MMAs)
+        ok = mbar_wait_sleep(&kfull, t & 1) && (t == 0 || mbar_wait_sleep(&ofull, (t - 1) & 1)) && !*abort_flag;
+        if (!ok) break;
         tc_fence_after();
-        const uint32_t q = smem_u32(sQ), k = smem_u32(sK(st));
 #pragma unroll
         for (int kk = 0; kk < kPaHD / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kPaHalf + (kk & 3) * 32;
-          tc_mma(tmem + kPaS0 + sb * kPaB, sdesc(q + off), sdesc(k + off), idesc_s, kk > 0 ? 1u : 0u);
+          tc_mma(tmem + kPaS, sdesc(q + off), sdesc(k + off), idesc_s, kk > 0 ? 1u : 0u);
         }
-        tc_commit(&sfull[sb]);
-        return true;
-      };
-      ok = ok && !*abort_flag && issue_s(0);
-      for (int t = 0; t < nt && ok; ++t) {
-        if (t + 1 < nt && !(ok = issue_s(t + 1))) break;
-        if (!(ok = mbar_wait(&pfull, t & 1)) || *abort_flag) {
-          ok = false;
-          break;
-        }
+        tc_commit(&sfull);
+        tc_commit(&kempty);
+        ok = mbar_wait_sleep(&pfull, t & 1) && mbar_wait_sleep(&vfull, t & 1) && !*abort_flag;
+        if (!ok) break;
         tc_fence_after();
-        const uint32_t v = smem_u32(sV(t & 1));
 #pragma unroll
         for (int kk = 0; kk < kPaB / 16; ++kk)  // 16 keys: two 8-row groups of the V tile
-          tc_mma_ts(tmem + kPaO, tmem + kPaP + kk * 8, sdesc_mn(v + kk * 2048, kPaHalf), idesc_o,
+          tc_mma_ts(tmem + kPaO, tmem + kPaS + kk * 8, sdesc_mn(v + kk * 2048, kPaHalf), idesc_o,
                     (t > 0 || kk > 0) ? 1u : 0u);
         tc_commit(&ofull);
-        tc_commit(&kvempty[t & 1]);
+        tc_commit(&vempty);
       }
       if (!ok) fail();
       tc_commit(&mma_done);
@@ -183,80 +211,92 @@ __global__ void __launch_bounds__(kPaThreads, 1)
     const int qrow = q0 + row;  // position in the sequence
     const uint32_t lane_base = tmem + ((uint32_t)(quad * 32) << 16);
     const float scale = kPaLog2e * rsqrtf((float)kPaHD);
-    float m = -INFINITY, l = 0.f;
+    float m = -INFINITY, l = 0.f;  // reference maximum (log2 domain) and row sum
     bool ok = true;
     for (int t = 0; t < nt; ++t) {
-      const int sb = t & 1;
-      ok = mbar_wait(&sfull[sb], (t >> 1) & 1);
+      ok = mbar_wait_sleep(&sfull, t & 1);
       if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      float s[kPaB];
-#pragma unroll
-      for (int c = 0; c < kPaB / 32; ++c) {
-        uint32_t r[32];
-        tc_ld<32>(lane_base + kPaS0 + sb * kPaB + c * 32, r);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) s[c * 32 + i] = __uint_as_float(r[i]);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sempty[sb]);
-
-      // scale, causal mask, running maximum (log2 domain)
       const int key0 = t * kPaB;
-      float mx = -INFINITY;
+      // keys past this row or past S only occur in the diagonal tile
+      const bool masked = key0 + kPaB - 1 > q0 || key0 + kPaB > S;
+      // raw scores of chunk c (32 columns); masked keys read -inf
+      auto load_raw = [&](auto mask, int c, float* v) {
+        uint32_t r[32];
+        tc_ld<32>(lane_base + kPaS + c * 32, r);
 #pragma unroll
-      for (int j = 0; j < kPaB; ++j) {
-        const int key = key0 + j;
-        const float v = (key > qrow || key >= S) ? -INFINITY : s[j] * scale;
-        s[j] = v;
-        mx = fmaxf(mx, v);
-      }
-      const float mnew = fmaxf(m, mx);
-      const float mref = mnew == -INFINITY ? 0.f : mnew;
-      const float corr = exp2f(m - mref);  // 0 on the first tile
-      float ps = 0.f;
-      uint32_t pw[kPaB / 2];
-#pragma unroll
-      for (int j = 0; j < kPaB; j += 2) {
-        const float p0 = exp2f(s[j] - mref), p1 = exp2f(s[j + 1] - mref);
-        ps += p0 + p1;
-        pw[j / 2] = pack_bf2(p0, p1);
-      }
-      l = l * corr + ps;
-      m = mnew;
-
-      if (t > 0) {
-        // the previous P V has completed: its P columns are free and O is final for it
-        ok = mbar_wait(&ofull, (t - 1) & 1);
-        if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        if (__any_sync(0xffffffffu, corr != 1.f)) {  // rescale O (warp-wide TMEM access)
-#pragma unroll 1
-          for (int c = 0; c < kPaHD / 32; ++c) {
-            uint32_t r[32];
-            tc_ld<32>(lane_base + kPaO + c * 32, r);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * corr);
-            tc_st32(lane_base + kPaO + c * 32, r);
+        for (int i = 0; i < 32; ++i) {
+          v[i] = __uint_as_float(r[i]);
+          if constexpr (decltype(mask)::value) {
+            const int key = key0 + c * 32 + i;
+            if (key > qrow || key >= S) v[i] = -INFINITY;
           }
         }
+      };
+      // pass 1: the row maximum of the raw scores (scale > 0 keeps the order)
+      auto row_max = [&](auto mask) {
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll 1
+        for (int c = 0; c < kPaB / 32; ++c) {
+          float v[32];
+          load_raw(mask, c, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) m4[i & 3] = fmaxf(m4[i & 3], v[i]);
+        }
+        return fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+      };
+      const float mraw = masked ? row_max(std::true_type{}) : row_max(std::false_type{});
+      const float mx = mraw * scale;
+      // move the reference when the tile would exceed it by more than 2^kPaSlack
+      float corr = 1.f;
+      if (mx > m + kPaSlack) {
+        corr = exp2f(m - mx);  // 0 on the first tile
+        m = mx;
+        l *= corr;
       }
-      tc_st32(lane_base + kPaP, pw);
-      tc_st32(lane_base + kPaP + 32, pw + 32);
+      if (t > 0 && __any_sync(0xffffffffu, corr != 1.f)) {
+        // O holds P V of the earlier tiles (complete: S(t) was issued after it)
+#pragma unroll 1
+        for (int c = 0; c < kPaHD / 32; ++c) {
+          uint32_t r[32];
+          tc_ld<32>(lane_base + kPaO + c * 32, r);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * corr);
+          tc_st32(lane_base + kPaO + c * 32, r);
+        }
+      }
+      // pass 2: P = 2^(s scale - m) as bf16 pairs over the score columns already read
+      const float mref = m == -INFINITY ? 0.f : m;
+      auto write_p = [&](auto mask) {
+        float p4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+        for (int c = 0; c < kPaB / 32; ++c) {
+          float v[32];
+          load_raw(mask, c, v);
+          uint32_t pw[16];
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            const float p0 = pa_ex2(fmaf(v[i], scale, -mref)), p1 = pa_ex2(fmaf(v[i + 1], scale, -mref));
+            p4[i & 3] += p0;
+            p4[(i + 1) & 3] += p1;
+            pw[i / 2] = pa_pack(p0, p1);
+          }
+          pa_st16(lane_base + kPaS + c * 16, pw);
+        }
+        return (p4[0] + p4[1]) + (p4[2] + p4[3]);
+      };
+      const float ps = masked ? write_p(std::true_type{}) : write_p(std::false_type{});
+      l += ps;
       tc_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull);
     }
     if (ok) {
-      ok = mbar_wait(&ofull, (nt - 1) & 1);
+      ok = mbar_wait_sleep(&ofull, (nt - 1) & 1);
       ok = __all_sync(0xffffffffu, ok);
     }
     if (ok) {
