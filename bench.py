@@ -86,27 +86,11 @@ def kernel_bytes(a, wq, kvq, B, ctx):
 # null.  Attention traffic is per cached token row (captured at B 8, context
 # 612) and scales with B x context.
 NCU_TRAFFIC = {
-    "attn": {"bytes": 81833472, "units": 8 * 612, "src": "fp_attention.cu", "sha": "95e873c98defbd20"},
+    "attn": {"bytes": 81739520, "units": 8 * 612, "src": "fp_attention.cu", "sha": "de945a405c820013"},
     "lm_head": {"bytes": 270745088, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
     "lin_gu": {"bytes": 94480640, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
     "lin_qkv": {"bytes": 50461184, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
     "lin_o": {"bytes": 16944384, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-}
-
-
-# ---------------------------------------------------------------- ncu traffic
-# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
-# 7B-shaped decode kernels from the ncu captures summarised in profiles/
-# (microbench cases 7b-*), with the sha256 prefix of the kernel's source at
-# capture time: a changed source makes the figure stale and it is reported as
-# null.  Attention traffic is per cached token row (captured at B 8, context
-# 612) and scales with B x context.
-NCU_TRAFFIC = {
-    "attn": {"bytes": 81945088, "units": 8 * 612, "src": "fp_attention.cu", "sha": "18124087fcad1249"},
-    "lm_head": {"bytes": 270379776, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
-    "lin_gu": {"bytes": 94771200, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
-    "lin_qkv": {"bytes": 50478848, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
-    "lin_o": {"bytes": 16944384, "units": None, "src": "fp_linear.cu", "sha": "6d8a772b845146d9"},
 }
 
 
