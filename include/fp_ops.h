@@ -151,7 +151,12 @@ int fp_op_attention_decode_noalloc(const uint16_t* q, int q_stride, int B, int n
 
 /* Prefill attention: causal, S query rows per sequence at positions 0..S-1,
  * q bf16 [B*S][q_stride]; keys/values read from the cache positions 0..S-1;
- * out bf16 [B*S][n_heads*head_dim]. */
+ * out bf16 [B*S][n_heads*head_dim].  head_dim 128 with 16-token pages,
+ * 16-byte aligned q (q_stride a multiple of 8) and pools runs on tcgen05
+ * (scores and output accumulated in TMEM); other shapes on mma.sync.  An
+ * int8 cache enters as its codes (exact in bf16), with each key's K scale
+ * multiplying its score column and its V scale its probability column in
+ * fp32.  A page id outside [0, n_pages) reads zeros and sets *err = 1. */
 int fp_op_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
                             const fp_kv_view* kv, uint16_t* out, int32_t* err, void* stream);
 

@@ -1,5 +1,5 @@
-// Prefill attention on the tcgen05 tensor cores: bf16 paged cache, head_dim
-// 128.
+// Prefill attention on the tcgen05 tensor cores: paged cache of bf16 or int8
+// codes with per-(token, KV head) fp32 scales, head_dim 128.
 //
 // o = softmax(q K^T / sqrt(hd) + causal mask) V for the S query rows of one
 // (sequence, head) against cache positions 0..S-1 (Sec. 5.1: the block's
@@ -7,10 +7,10 @@
 // CTAs per SM (256 TMEM columns and 97 KiB of shared memory each), so one
 // CTA's softmax overlaps the other's MMAs and loads:
 //   warp 0      TMA: the Q tile once (two 64-column boxes of the q rows), then
-//               per key tile its K rows and its V rows page by page (a
-//               [16][64] box per 16-token page and half of head_dim, 128-byte
-//               swizzle); K(t + 1) loads once S(t) has read K(t), V(t + 1)
-//               once P(t) V(t) has read V(t);
+//               (bf16 cache) per key tile its K rows and its V rows page by
+//               page (a [16][64] box per 16-token page and half of head_dim,
+//               128-byte swizzle); K(t + 1) loads once S(t) has read K(t),
+//               V(t + 1) once P(t) V(t) has read V(t);
 //   warp 1      allocates the TMEM and issues the MMAs: S = Q K^T (M 128
 //               queries, N 128 keys, K 16 over head_dim; K-major operands),
 //               then O += P V (A = P from TMEM, B = V read MN-major);
@@ -20,6 +20,13 @@
 //               already read.  The reference maximum m only moves when a tile
 //               raises it by more than 2^8 (O and the row sum are rescaled
 //               then); P never exceeds 256, and o / l is exact either way.
+//   int8 cache: warps 0, 6 and 7 (after warp 0 has issued the Q copy) widen
+//               the codes: each loads its rows' 16-byte code chunks, turns
+//               them into bf16 (integers of at most 8 bits: exact) in the
+//               same swizzled layout the TMA writes, and stages the tile's K
+//               and V scales; the softmax multiplies each score column by
+//               its K scale and each P column by its V scale (the row sum
+//               takes the unscaled P), so the scales enter in fp32.
 // TMEM columns: scores S [0, 128) with P over [0, 64), O [128, 256).  Every
 // mbarrier wait is bounded (error 2 past the limit); a page id out of range
 // reads zeros and sets error 1.
@@ -34,13 +41,19 @@ namespace fpk {
 
 constexpr int kPaB = 128;  // query rows per CTA = keys per tile
 constexpr int kPaHD = 128;
-constexpr int kPaThreads = 192;
+constexpr int kPaWiden = 3;                                 // int8 cache: warps widening codes (0, 6, 7)
+constexpr int kPaWRows = (kPaB + 4 * kPaWiden - 1) / (4 * kPaWiden);  // tile rows per widening thread
+template <bool KV8>
+constexpr int pa_threads() { return KV8 ? 256 : 192; }
 constexpr uint32_t kPaTmemCols = 256;
 constexpr uint32_t kPaS = 0, kPaO = 128;
 constexpr int kPaHalf = kPaB * 128;          // bytes of one [128 rows][64 bf16] swizzled half
 constexpr int kPaTile = 2 * kPaHalf;         // one [128][128] bf16 operand
 constexpr int kPaSmem = 3 * kPaTile + 1024;  // Q, K, V, alignment
 constexpr float kPaLog2e = 1.4426950408889634f;
+// score columns per TMEM load in the softmax (64-column loads measured
+// slower: 201 / 319 against 211 / 356 TFLOP/s at the 7B / 13B shapes)
+constexpr int kPaCW = 32;
 constexpr float kPaSlack = 8.f;  // log2 of the largest P allowed before the reference maximum moves
 
 // Shared-memory descriptor of an MN-major operand with 128-byte swizzle:
@@ -74,15 +87,25 @@ FP_DEV uint32_t pa_pack(float lo, float hi) {
   return r;
 }
 
-__global__ void __launch_bounds__(kPaThreads, 2)
+// Signed byte `i` (0..3) of `w` as an exact fp32: 2^23 + (byte ^ 0x80) built
+// by a byte permute, then the offset subtracted.
+FP_DEV float pa_i8f(uint32_t w, int i) {
+  return __uint_as_float(__byte_perm(w ^ 0x80808080u, 0x4B000000u, 0x7650 | i)) - 8388736.f;
+}
+
+template <bool KV8>
+__global__ void __launch_bounds__(pa_threads<KV8>(), 2)
     attn_prefill_tc_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                           const __grid_constant__ CUtensorMap map_v, int S, int H, int Hkv, int page_size,
+                           const __grid_constant__ CUtensorMap map_v, const int8_t* __restrict__ k8,
+                           const int8_t* __restrict__ v8, const float* __restrict__ k_scale,
+                           const float* __restrict__ v_scale, int S, int H, int Hkv, int page_size,
                            const int32_t* __restrict__ page_table, int pages_per_seq, int n_pages,
                            uint16_t* __restrict__ out, int32_t* err) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint64_t qfull, kfull, kempty, vfull, vempty, sfull, pfull, ofull, mma_done;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_word;
+  __shared__ __align__(16) float s_scl[KV8 ? 4 * kPaB : 4];  // int8: [K, V][tile parity][key] scales
   volatile int* abort_flag = &abort_word;
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sQ = smem;
@@ -101,9 +124,9 @@ __global__ void __launch_bounds__(kPaThreads, 2)
   pdl_trigger();
   if (threadIdx.x == 0) {
     mbar_init(&qfull, 1);
-    mbar_init(&kfull, 1);
+    mbar_init(&kfull, KV8 ? kPaWiden : 1);
     mbar_init(&kempty, 1);
-    mbar_init(&vfull, 1);
+    mbar_init(&vfull, KV8 ? kPaWiden : 1);
     mbar_init(&vempty, 1);
     mbar_init(&sfull, 1);
     mbar_init(&pfull, 4);
@@ -124,7 +147,89 @@ __global__ void __launch_bounds__(kPaThreads, 2)
   const uint32_t tmem = tmem_base;
   pdl_wait();
 
-  if (warp == 0) {
+  if (KV8 && (warp == 0 || warp >= 6)) {
+    // ---------------- int8 cache: the Q copy, then widening of the key tiles
+    if (warp == 0 && lane == 0) {
+      mbar_expect_tx(&qfull, kPaTile);
+      tma_load_2d(sQ, &map_q, h * kPaHD, b * S + q0, &qfull);
+      tma_load_2d(sQ + kPaHalf, &map_q, h * kPaHD + 64, b * S + q0, &qfull);
+    }
+    const int wi = (warp == 0 ? 0 : warp - 5) * 32 + lane;  // 0 .. 95
+    const int c = wi & 7;                                     // code chunk: head_dim 16c .. 16c + 15
+    const int rbase = wi >> 3;                                // tile rows rbase + 12i (< 128)
+    // its bf16 form is chunks cb, cb + 1 of half c / 4 of the swizzled row;
+    // the lanes of the upper half store the odd chunk first, so the eight
+    // lanes of one row write eight distinct 16-byte bank groups
+    const int cb = 2 * (c & 3), half_off = (c >> 2) * kPaHalf;
+    const int32_t* pt = page_table + (long long)b * pages_per_seq;
+    bool ok = true;
+    for (int t = 0; t < nt && ok; ++t) {
+      int rowi[kPaWRows];  // pool row of each of the thread's keys (< 2^31); -1 reads zeros
+#pragma unroll
+      for (int i = 0; i < kPaWRows; ++i) {
+        const int row = rbase + 4 * kPaWiden * i, key = t * kPaB + row;
+        rowi[i] = -1;
+        if (row < kPaB && key < S) {
+          const int pg = __ldg(pt + key / page_size);
+          if (pg >= 0 && pg < n_pages) rowi[i] = (pg * Hkv + kvh) * page_size + key % page_size;
+          else if (err && c == 0) atomicExch(err, 1);
+        }
+      }
+      // the tile's K and V scales go out with its K codes: the softmax reads
+      // both once S(t) is complete, which only the K tile's barrier precedes
+      float sck[kPaWRows], scv[kPaWRows];
+#pragma unroll
+      for (int i = 0; i < kPaWRows; ++i) {
+        sck[i] = (c == 0 && rowi[i] >= 0) ? __ldg(k_scale + rowi[i]) : 0.f;
+        scv[i] = (c == 0 && rowi[i] >= 0) ? __ldg(v_scale + rowi[i]) : 0.f;
+      }
+#pragma unroll 1
+      for (int which = 0; which < 2; ++which) {
+        const int8_t* pool = which ? v8 : k8;
+        uint4 w[kPaWRows];
+        // the codes are read before the wait for the buffer
+#pragma unroll
+        for (int i = 0; i < kPaWRows; ++i)
+          w[i] = rowi[i] >= 0 ? ld_nc16(pool + (long long)rowi[i] * kPaHD + c * 16) : make_uint4(0, 0, 0, 0);
+        ok = t == 0 || mbar_wait_sleep(which ? &vempty : &kempty, (t - 1) & 1);
+        if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
+          ok = false;
+          break;
+        }
+        uint8_t* dst = (which ? sV : sK) + half_off;
+#pragma unroll
+        for (int i = 0; i < kPaWRows; ++i) {
+          const int row = rbase + 4 * kPaWiden * i, sw = row & 7;
+          if (row >= kPaB) break;
+          const uint32_t ww[4] = {w[i].x, w[i].y, w[i].z, w[i].w};
+          uint32_t o[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            o[j] = pa_pack(pa_i8f(ww[j >> 1], (2 * j) & 3), pa_i8f(ww[j >> 1], (2 * j + 1) & 3));
+          const uint4 e = make_uint4(o[0], o[1], o[2], o[3]), f = make_uint4(o[4], o[5], o[6], o[7]);
+          uint8_t* rp = dst + row * 128;
+          if (c < 4) {
+            *reinterpret_cast<uint4*>(rp + ((cb ^ sw) << 4)) = e;
+            *reinterpret_cast<uint4*>(rp + (((cb + 1) ^ sw) << 4)) = f;
+          } else {
+            *reinterpret_cast<uint4*>(rp + (((cb + 1) ^ sw) << 4)) = f;
+            *reinterpret_cast<uint4*>(rp + ((cb ^ sw) << 4)) = e;
+          }
+          if (which == 0 && c == 0) {
+            // buffer t & 1 was last read by the softmax of tile t - 2, which
+            // completed before S(t - 1) was issued and so before this K tile's wait
+            s_scl[(t & 1) * kPaB + row] = sck[i];
+            s_scl[(2 + (t & 1)) * kPaB + row] = scv[i];
+          }
+        }
+        fence_proxy_async();  // the MMAs read the tile through the async proxy
+        __syncwarp();
+        if (lane == 0) mbar_arrive(which ? &vfull : &kfull);
+      }
+    }
+    if (!ok && lane == 0) fail();
+    if (warp == 0 && lane == 0) mbar_wait(&qfull, 0);  // the Q copy lands before the CTA leaves
+  } else if (warp == 0) {
     // ---------------- TMA producer
     if (lane == 0) {
       const int32_t* pt = page_table + (long long)b * pages_per_seq;
@@ -223,15 +328,27 @@ __global__ void __launch_bounds__(kPaThreads, 2)
       const int key0 = t * kPaB;
       // keys past this row or past S only occur in the diagonal tile
       const bool masked = key0 + kPaB - 1 > q0 || key0 + kPaB > S;
-      // raw scores of chunk c (32 columns); masked keys read -inf
+      // raw scores of chunk c (kPaCW columns); masked keys read -inf
       auto load_raw = [&](auto mask, int c, float* v) {
-        uint32_t r[32];
-        tc_ld<32>(lane_base + kPaS + c * 32, r);
+        uint32_t r[kPaCW];
+        tc_ld<kPaCW>(lane_base + kPaS + c * kPaCW, r);
+        if constexpr (KV8) {
+          // K scale of each key column (masked columns are overwritten below)
+          const float4* k4 = reinterpret_cast<const float4*>(s_scl + (t & 1) * kPaB + c * kPaCW);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
+          for (int i = 0; i < kPaCW / 4; ++i) {
+            const float4 f = k4[i];
+            r[4 * i] = __float_as_uint(__uint_as_float(r[4 * i]) * f.x);
+            r[4 * i + 1] = __float_as_uint(__uint_as_float(r[4 * i + 1]) * f.y);
+            r[4 * i + 2] = __float_as_uint(__uint_as_float(r[4 * i + 2]) * f.z);
+            r[4 * i + 3] = __float_as_uint(__uint_as_float(r[4 * i + 3]) * f.w);
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < kPaCW; ++i) {
           v[i] = __uint_as_float(r[i]);
           if constexpr (decltype(mask)::value) {
-            const int key = key0 + c * 32 + i;
+            const int key = key0 + c * kPaCW + i;
             if (key > qrow || key >= S) v[i] = -INFINITY;
           }
         }
@@ -240,11 +357,11 @@ __global__ void __launch_bounds__(kPaThreads, 2)
       auto row_max = [&](auto mask) {
         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll 1
-        for (int c = 0; c < kPaB / 32; ++c) {
-          float v[32];
+        for (int c = 0; c < kPaB / kPaCW; ++c) {
+          float v[kPaCW];
           load_raw(mask, c, v);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) m4[i & 3] = fmaxf(m4[i & 3], v[i]);
+          for (int i = 0; i < kPaCW; ++i) m4[i & 3] = fmaxf(m4[i & 3], v[i]);
         }
         return fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
       };
@@ -273,18 +390,24 @@ __global__ void __launch_bounds__(kPaThreads, 2)
       auto write_p = [&](auto mask) {
         float p4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll 1
-        for (int c = 0; c < kPaB / 32; ++c) {
-          float v[32];
+        for (int c = 0; c < kPaB / kPaCW; ++c) {
+          float v[kPaCW];
           load_raw(mask, c, v);
-          uint32_t pw[16];
+          uint32_t pw[kPaCW / 2];
 #pragma unroll
-          for (int i = 0; i < 32; i += 2) {
+          for (int i = 0; i < kPaCW; i += 2) {
             const float p0 = pa_ex2(fmaf(v[i], scale, -mref)), p1 = pa_ex2(fmaf(v[i + 1], scale, -mref));
             p4[i & 3] += p0;
             p4[(i + 1) & 3] += p1;
-            pw[i / 2] = pa_pack(p0, p1);
+            if constexpr (KV8) {
+              // V scale of each key column: P V then takes the codes as they are
+              const float2 vs = *reinterpret_cast<const float2*>(s_scl + (2 + (t & 1)) * kPaB + c * kPaCW + i);
+              pw[i / 2] = pa_pack(p0 * vs.x, p1 * vs.y);
+            } else {
+              pw[i / 2] = pa_pack(p0, p1);
+            }
           }
-          pa_st16(lane_base + kPaS + c * 16, pw);
+          pa_st16(lane_base + kPaS + c * (kPaCW / 2), pw);
         }
         return (p4[0] + p4[1]) + (p4[2] + p4[3]);
       };
@@ -330,29 +453,41 @@ __global__ void __launch_bounds__(kPaThreads, 2)
 }
 
 bool attention_prefill_tc_ok(int B, int S, int n_heads, const fp_kv_view& kv, const void* q, int q_stride) {
-  return kv.kvquant == FP_KV_BF16 && kv.head_dim == kPaHD && kv.page_size == 16 && B >= 1 && S >= 1 &&
-         n_heads % kv.n_kv_heads == 0 && q_stride % 8 == 0 && ((uintptr_t)q & 15) == 0 &&
-         ((uintptr_t)kv.k_pool & 15) == 0 && ((uintptr_t)kv.v_pool & 15) == 0 &&
+  const bool kv8 = kv.kvquant == FP_KV_INT8;
+  return (kv.kvquant == FP_KV_BF16 || (kv8 && kv.k_scale && kv.v_scale)) && kv.head_dim == kPaHD &&
+         kv.page_size == 16 && B >= 1 && S >= 1 && n_heads % kv.n_kv_heads == 0 && q_stride % 8 == 0 &&
+         ((uintptr_t)q & 15) == 0 && ((uintptr_t)kv.k_pool & 15) == 0 && ((uintptr_t)kv.v_pool & 15) == 0 &&
          (long long)kv.n_pages * kv.n_kv_heads * kv.page_size < (1LL << 31) && tensor_maps_available();
+}
+
+template <bool KV8>
+static cudaError_t launch_pa_tc(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv, int B, int S,
+                                int n_heads, const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s) {
+  static bool attr = false;
+  if (!attr) {
+    FP_CUDA_TRY(
+        cudaFuncSetAttribute(attn_prefill_tc_kernel<KV8>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPaSmem));
+    attr = true;
+  }
+  const dim3 grid((S + kPaB - 1) / kPaB, n_heads, B);
+  return launch(attn_prefill_tc_kernel<KV8>, grid, dim3(pa_threads<KV8>()), (size_t)kPaSmem, s, mq, mk, mv,
+                (const int8_t*)kv.k_pool, (const int8_t*)kv.v_pool, (const float*)kv.k_scale,
+                (const float*)kv.v_scale, S, n_heads, kv.n_kv_heads, kv.page_size, kv.page_table, kv.pages_per_seq,
+                kv.n_pages, out, err);
 }
 
 cudaError_t launch_attention_prefill_tc(const uint16_t* q, int q_stride, int B, int S, int n_heads,
                                         const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s) {
   CUtensorMap mq, mk, mv;
   const long long pool_rows = (long long)kv.n_pages * kv.n_kv_heads * kv.page_size;
-  // q [B S][q_stride] bf16, box [128 rows][64]; pools [pages Hkv 16][128] bf16, box [16 rows][64]
-  if (!make_tensor_map(&mq, q, (long long)B * S, q_stride, 2, kPaB, 64, 128) ||
-      !make_tensor_map(&mk, kv.k_pool, pool_rows, kPaHD, 2, 16, 64, 128) ||
+  // q [B S][q_stride] bf16, box [128 rows][64]
+  if (!make_tensor_map(&mq, q, (long long)B * S, q_stride, 2, kPaB, 64, 128)) return cudaErrorInvalidValue;
+  if (kv.kvquant == FP_KV_INT8) return launch_pa_tc<true>(mq, mq, mq, B, S, n_heads, kv, out, err, s);
+  // bf16 pools [pages Hkv 16][128], box [16 rows][64]
+  if (!make_tensor_map(&mk, kv.k_pool, pool_rows, kPaHD, 2, 16, 64, 128) ||
       !make_tensor_map(&mv, kv.v_pool, pool_rows, kPaHD, 2, 16, 64, 128))
     return cudaErrorInvalidValue;
-  static bool attr = false;
-  if (!attr) {
-    FP_CUDA_TRY(cudaFuncSetAttribute(attn_prefill_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kPaSmem));
-    attr = true;
-  }
-  const dim3 grid((S + kPaB - 1) / kPaB, n_heads, B);
-  return launch(attn_prefill_tc_kernel, grid, dim3(kPaThreads), (size_t)kPaSmem, s, mq, mk, mv, S, n_heads,
-                kv.n_kv_heads, kv.page_size, kv.page_table, kv.pages_per_seq, kv.n_pages, out, err);
+  return launch_pa_tc<false>(mq, mk, mv, B, S, n_heads, kv, out, err, s);
 }
 
 }  // namespace fpk

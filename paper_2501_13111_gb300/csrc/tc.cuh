@@ -102,6 +102,9 @@ FP_DEV void tc_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
                : "memory");
 }
+// Orders this thread's generic-proxy shared-memory writes before later
+// async-proxy reads (tcgen05.mma operands, TMA stores) of the same bytes.
+FP_DEV void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 FP_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 FP_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 
@@ -114,7 +117,7 @@ FP_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;
 // wait for the load sits in the same asm statement as the load: the
 // destination registers are undefined until tcgen05.wait::ld, and a separate
 // statement would not stop the compiler from reading them before it.
-// N = 4, 8, 16 or 32.
+// N = 4, 8, 16, 32 or 64.
 template <int N>
 FP_DEV void tc_ld(uint32_t taddr, uint32_t* r) {
   if constexpr (N == 4) {
@@ -138,8 +141,17 @@ FP_DEV void tc_ld(uint32_t taddr, uint32_t* r) {
         : FP_R8(0), FP_R8(8)
         : "r"(taddr)
         : "memory");
+  } else if constexpr (N == 64) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+        "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,"
+        "%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : FP_R8(0), FP_R8(8), FP_R8(16), FP_R8(24), FP_R8(32), FP_R8(40), FP_R8(48), FP_R8(56)
+        : "r"(taddr)
+        : "memory");
   } else {
-    static_assert(N == 32, "tc_ld: 4, 8, 16 or 32 columns");
+    static_assert(N == 32, "tc_ld: 4, 8, 16, 32 or 64 columns");
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
         "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
