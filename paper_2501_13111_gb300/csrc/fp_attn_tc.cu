@@ -9,8 +9,8 @@
 //   warp 0      TMA: the Q tile once (two 64-column boxes of the q rows), then
 //               (bf16 cache) per key tile its K rows and its V rows page by
 //               page (a [16][64] box per 16-token page and half of head_dim,
-//               128-byte swizzle); K(t + 1) loads once S(t) has read K(t),
-//               V(t + 1) once P(t) V(t) has read V(t);
+//               128-byte swizzle, one box per lane); K(t + 1) loads once S(t)
+//               has read K(t), V(t + 1) once P(t) V(t) has read V(t);
 //   warp 1      allocates the TMEM and issues the MMAs: S = Q K^T (M 128
 //               queries, N 128 keys, K 16 over head_dim; K-major operands),
 //               then O += P V (A = P from TMEM, B = V read MN-major);
@@ -191,7 +191,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
 #pragma unroll
         for (int i = 0; i < kPaWRows; ++i)
           w[i] = rowi[i] >= 0 ? ld_nc16(pool + (long long)rowi[i] * kPaHD + c * 16) : make_uint4(0, 0, 0, 0);
-        ok = t == 0 || mbar_wait_sleep(which ? &vempty : &kempty, (t - 1) & 1);
+        ok = t == 0 || mbar_wait(which ? &vempty : &kempty, (t - 1) & 1);
         if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
           ok = false;
           break;
@@ -230,48 +230,56 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
     if (!ok && lane == 0) fail();
     if (warp == 0 && lane == 0) mbar_wait(&qfull, 0);  // the Q copy lands before the CTA leaves
   } else if (warp == 0) {
-    // ---------------- TMA producer
+    // ---------------- TMA producer: lanes 0-15 each copy one [16][64] box of
+    // a key tile (page lane & 7, head_dim half lane >> 3); lane 0 arms the
+    // barriers.  The next tile's page ids are read while this one is in flight.
+    const int32_t* pt = page_table + (long long)b * pages_per_seq;
+    const int pg = lane & 7, half = (lane >> 3) & 1;
+    auto page_row = [&](int t) {  // pool row of this lane's page of tile t; -16 reads zeros
+      const int key0 = t * kPaB + pg * 16;
+      if (lane >= 16 || key0 >= S) return -16;
+      const int id = __ldg(pt + key0 / page_size);
+      if (id >= 0 && id < n_pages) return (id * Hkv + kvh) * page_size;
+      if (err && half == 0) atomicExch(err, 1);
+      return -16;
+    };
     if (lane == 0) {
-      const int32_t* pt = page_table + (long long)b * pages_per_seq;
-      // the key tile's rows, page by page (rows past S, or of a bad page, read zeros)
-      auto load_rows = [&](const CUtensorMap* map, uint8_t* dst, int t, uint64_t* bar) {
-        int rows[kPaB / 16];  // the page ids are all read before the first copy is issued
-#pragma unroll
-        for (int pg = 0; pg < kPaB / 16; ++pg) {
-          const int key0 = t * kPaB + pg * 16;
-          rows[pg] = key0 < S ? __ldg(pt + key0 / page_size) : -1;
-        }
-#pragma unroll
-        for (int pg = 0; pg < kPaB / 16; ++pg) {
-          int row = -16;
-          if (t * kPaB + pg * 16 < S) {
-            if (rows[pg] >= 0 && rows[pg] < n_pages) row = (rows[pg] * Hkv + kvh) * page_size;
-            else if (err) atomicExch(err, 1);
-          }
-          tma_load_2d(dst + pg * 2048, map, 0, row, bar);
-          tma_load_2d(dst + kPaHalf + pg * 2048, map, 64, row, bar);
-        }
-      };
+      asm volatile("prefetch.tensormap [%0];" ::"l"(&map_k) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(&map_v) : "memory");
       mbar_expect_tx(&qfull, kPaTile);
       tma_load_2d(sQ, &map_q, h * kPaHD, b * S + q0, &qfull);
       tma_load_2d(sQ + kPaHalf, &map_q, h * kPaHD + 64, b * S + q0, &qfull);
-      int kiss = 0, viss = 0;
-      for (int t = 0; t < nt; ++t) {
-        if (t > 0 && (!mbar_wait_sleep(&kempty, (t - 1) & 1) || *abort_flag)) {
-          fail();
+    }
+    int row = page_row(0);
+    int kiss = 0, viss = 0;
+    bool ok = true;
+    for (int t = 0; t < nt; ++t) {
+      if (t > 0) {
+        ok = mbar_wait(&kempty, (t - 1) & 1);
+        if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
+          ok = false;
           break;
         }
-        mbar_expect_tx(&kfull, kPaTile);
-        load_rows(&map_k, sK, t, &kfull);
-        kiss = t + 1;
-        if (t > 0 && (!mbar_wait_sleep(&vempty, (t - 1) & 1) || *abort_flag)) {
-          fail();
-          break;
-        }
-        mbar_expect_tx(&vfull, kPaTile);
-        load_rows(&map_v, sV, t, &vfull);
-        viss = t + 1;
       }
+      if (lane == 0) mbar_expect_tx(&kfull, kPaTile);
+      __syncwarp();
+      if (lane < 16) tma_load_2d(sK + half * kPaHalf + pg * 2048, &map_k, half * 64, row, &kfull);
+      kiss = t + 1;
+      if (t > 0) {
+        ok = mbar_wait(&vempty, (t - 1) & 1);
+        if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
+          ok = false;
+          break;
+        }
+      }
+      if (lane == 0) mbar_expect_tx(&vfull, kPaTile);
+      __syncwarp();
+      if (lane < 16) tma_load_2d(sV + half * kPaHalf + pg * 2048, &map_v, half * 64, row, &vfull);
+      viss = t + 1;
+      if (t + 1 < nt) row = page_row(t + 1);
+    }
+    if (lane == 0) {
+      if (!ok) fail();
       // copies still in flight land before the CTA leaves
       mbar_wait(&qfull, 0);
       if (kiss > 0) mbar_wait(&kfull, (kiss - 1) & 1);
@@ -282,11 +290,11 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
     if (lane == 0) {
       constexpr uint32_t idesc_s = tc_idesc(kPaB, kPaB);                // Q, K both K-major
       constexpr uint32_t idesc_o = tc_idesc(kPaB, kPaHD) | (1u << 16);  // V MN-major
-      bool ok = mbar_wait_sleep(&qfull, 0);
+      bool ok = mbar_wait(&qfull, 0);
       const uint32_t q = smem_u32(sQ), k = smem_u32(sK), v = smem_u32(sV);
       for (int t = 0; t < nt && ok; ++t) {
         // S(t) overwrites P(t - 1): its P V has completed (in order with this thread's MMAs)
-        ok = mbar_wait_sleep(&kfull, t & 1) && (t == 0 || mbar_wait_sleep(&ofull, (t - 1) & 1)) && !*abort_flag;
+        ok = mbar_wait(&kfull, t & 1) && (t == 0 || mbar_wait(&ofull, (t - 1) & 1)) && !*abort_flag;
         if (!ok) break;
         tc_fence_after();
 #pragma unroll
@@ -296,7 +304,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
         }
         tc_commit(&sfull);
         tc_commit(&kempty);
-        ok = mbar_wait_sleep(&pfull, t & 1) && mbar_wait_sleep(&vfull, t & 1) && !*abort_flag;
+        ok = mbar_wait(&pfull, t & 1) && mbar_wait(&vfull, t & 1) && !*abort_flag;
         if (!ok) break;
         tc_fence_after();
 #pragma unroll
@@ -319,7 +327,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
     float m = -INFINITY, l = 0.f;  // reference maximum (log2 domain) and row sum
     bool ok = true;
     for (int t = 0; t < nt; ++t) {
-      ok = mbar_wait_sleep(&sfull, t & 1);
+      ok = mbar_wait(&sfull, t & 1);
       if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
         ok = false;
         break;
@@ -419,7 +427,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
       if (lane == 0) mbar_arrive(&pfull);
     }
     if (ok) {
-      ok = mbar_wait_sleep(&ofull, (nt - 1) & 1);
+      ok = mbar_wait(&ofull, (nt - 1) & 1);
       ok = __all_sync(0xffffffffu, ok);
     }
     if (ok) {
