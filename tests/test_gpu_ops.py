@@ -290,6 +290,55 @@ def test_attention_prefill(fp, kvq, hd, H, Hkv, S):
 
 
 @pytest.mark.parametrize("kvq", [0, 1])
+@pytest.mark.parametrize("hd,H,Hkv", [(64, 4, 4), (128, 8, 2)])
+def test_attention_bad_page_reads_zeros(fp, kvq, hd, H, Hkv):
+    """A page id outside [0, n_pages) reads as zero keys and values (zero
+    codes and scales for int8) and sets the error word to 1, in prefill and
+    in decode; the other pages are unaffected."""
+    B, S = 2, 200
+    c = Cache(fp, kvq, B, S + 5, Hkv, hd, seed=77 + hd + kvq)
+    bad = {(0, 5): c.n_pages, (1, 9): -3}  # positions 80-95 of sequence 0, 144-159 of sequence 1
+    table = c.table.copy()
+    for (b, pg), v in bad.items():
+        table[b, pg] = v
+    td = dev(table)
+    view = fp.fp_kv_view(kvq, Hkv, hd, c.P, c.pps, c.n_pages, ptr(c.kd), ptr(c.vd), ptr(c.ks), ptr(c.vs), ptr(td))
+
+    def seq(which, b, T):
+        x = c.seq(which, b, T)
+        for (bb, pg) in bad:
+            if bb == b:
+                x[pg * 16:(pg + 1) * 16] = 0.0
+        return x
+
+    q = synth.uniform_bf16(43, hd, (B * S, H * hd), -2, 2)
+    qf = quant.bf16_to_f32(q).astype(np.float64).reshape(B, S, H, hd)
+    out = empty(B * S * H * hd, np.uint16)
+    err = empty(1, np.int32)
+    fp.fp_op_attention_prefill(ptr(dev(q)), H * hd, B, S, H, view, ptr(out), ptr(err))
+    got = quant.bf16_to_f32(host(out, np.uint16)).reshape(B, S, H, hd)
+    for b in range(B):
+        ref = M.attention(qf[b], np.arange(S), seq("k", b, S), seq("v", b, S))
+        assert rel_err(got[b], ref) <= TAU[0] / 2, ("prefill", b, rel_err(got[b], ref))
+    assert host(err, np.int32)[0] == 1
+
+    lens = [S, 150]
+    qd = synth.uniform_bf16(44, hd, (B, H * hd), -2, 2)
+    wsb = fp.fp_op_attention_decode_workspace_bytes(B, H, hd, S + 5)
+    ws = empty(wsb)
+    out = empty(B * H * hd, np.uint16)
+    err = empty(1, np.int32)
+    fp.fp_op_attention_decode(ptr(dev(qd)), H * hd, B, H, view, ptr(dev(np.array(lens, np.int32))), S + 5, ptr(out),
+                              ptr(ws), wsb, ptr(err))
+    got = quant.bf16_to_f32(host(out, np.uint16)).reshape(B, H, hd)
+    qf = quant.bf16_to_f32(qd).astype(np.float64).reshape(B, H, hd)
+    for b, L in enumerate(lens):
+        ref = M.attention(qf[b][None], np.array([L - 1]), seq("k", b, L), seq("v", b, L))[0]
+        assert rel_err(got[b], ref) <= TAU[0] / 2, ("decode", b, rel_err(got[b], ref))
+    assert host(err, np.int32)[0] == 1
+
+
+@pytest.mark.parametrize("kvq", [0, 1])
 @pytest.mark.parametrize("hd", [64, 128])
 def test_rope_kv_write(fp, kvq, hd):
     B, S, H, Hkv, T = 3, 5, 4, 2, 48
