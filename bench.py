@@ -163,11 +163,12 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- oracle timing
-def oracle_sample(cfg, batch, steps, decode_tokens):
+def oracle_sample(cfg, batch, steps, decode_tokens, warmup=0):
     """Time the oracle (numpy fp64, test infrastructure) on the same workload:
     the full config shape at the same batch and prompt; the prompt's prefill
-    is set-up, each timed step is ``decode_tokens`` greedy decode steps.
-    Returns (tokens/s, seconds per step list, description)."""
+    is set-up, each step is ``decode_tokens`` greedy decode steps, the first
+    ``warmup`` steps untimed.  Returns (tokens/s, seconds per timed step,
+    description)."""
     import synth
     from oracle import model as M
 
@@ -176,19 +177,20 @@ def oracle_sample(cfg, batch, steps, decode_tokens):
     get = lambda l, k, shape: (synth.f32_to_bf16_bits(np.ones(shape, np.float32)) if len(shape) == 1
                                else synth.weight_bf16(0, l, k, shape))
     w, _ = M.build_weights(arch, wq, get)
-    ref = M.Fingerprint(arch, w, kvq, batch, S + steps * decode_tokens + 1)
+    ref = M.Fingerprint(arch, w, kvq, batch, S + (warmup + steps) * decode_tokens + 1)
     toks = synth.tokens(0, batch * S, arch.vocab).reshape(batch, S)
     out = ref.prefill(toks)
     tok = out["tokens"]
     times = []
-    for _ in range(steps):
+    for _ in range(warmup + steps):
         t0 = time.perf_counter()
         for _ in range(decode_tokens):
             tok = ref.decode(tok)["tokens"]
         times.append(time.perf_counter() - t0)
+    times = times[warmup:]
     tps = batch * decode_tokens * steps / sum(times)
     desc = (f"oracle decode, batch {batch}, prompt {S} (prefill untimed), {decode_tokens} tokens x {steps} "
-            f"timed steps, fp64 numpy")
+            f"timed steps" + (f" after {warmup} untimed" if warmup else "") + ", fp64 numpy")
     return tps, times, desc
 
 
@@ -209,9 +211,7 @@ def run_reference(args, cfg):
     if int(os.environ.get("RANK", "0")) != 0:
         return 0
     t, wq, kvq, B, S, N = cfg
-    tps, times, desc = oracle_sample(cfg, B, args.warmup + args.steps, 2)
-    times = times[args.warmup:]
-    tps = B * 2 * len(times) / sum(times)
+    tps, times, desc = oracle_sample(cfg, B, args.steps, 2, warmup=args.warmup)
     line = {
         "metric": METRIC, "value": tps, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
