@@ -1,0 +1,58 @@
+"""The bench's JSON line, checked on the host: the reference arm (the oracle
+timed on the host cores) on the tiny configuration, run as the driver runs it,
+and the kernel byte model that the roofline divides by."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+from tests.conftest import ROOT
+
+
+def _run_bench(*args):
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), *args], cwd=ROOT, env=env,
+                       capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout[-2000:]
+    return json.loads(lines[0])
+
+
+def test_reference_arm_line():
+    d = _run_bench("--impl", "reference", "--config", "tiny", "--steps", "2", "--warmup", "1")
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+              "vs_baseline", "dtype", "data", "config", "impl", "cpu_baseline", "e2e"):
+        assert k in d, k
+    assert d["impl"] == "reference" and d["steps"] == 2 and d["warmup"] == 1 and d["n_gpus"] == 1
+    assert d["unit"] == "tokens/s" and d["higher_is_better"] is True and d["value"] > 0
+    assert d["config"]["workload"] == "tiny-shaped fingerprint"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and "2 timed steps" in cb["sample"]
+    e = d["e2e"]
+    assert e["value"] == d["value"] and e["unit"] == d["unit"]
+    assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+    # tokens/s = batch x 2 tokens per step / mean step time
+    B = d["config"]["batch"]
+    assert abs(d["value"] - B * 2 / (d["ms_per_step"] * 1e-3)) <= 1e-6 * d["value"]
+
+
+def test_kernel_bytes_closed_forms():
+    """Algorithmic bytes per launch of the 7B-shaped decode classes, written
+    out from the weight formats (int8: N K codes + 2 N scales) and the
+    activations each launch reads and writes."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    t, wq, kvq, B, S, N = bench.CONFIGS["l7b"]
+    a = bench.arch_dict(t)
+    kb = bench.kernel_bytes(a, wq, kvq, B, S)
+    d, f, V = a["hidden"], a["ffn"], a["vocab"]
+    qkv = (a["n_heads"] + 2 * a["n_kv_heads"]) * a["head_dim"]
+    assert kb["lin_qkv"] == qkv * d + 2 * qkv + 2 * B * (d + qkv)
+    assert kb["lin_gu"] == 2 * f * d + 2 * 2 * f + 2 * B * (d + f)
+    assert kb["lm_head"] == 2 * V * d + 2 * B * d + 4 * B * V
+    # one block's K and V: B x context x Hkv x hd x 2 (K and V) x 2 bytes
+    assert kb["attn"] == pytest.approx(B * S * a["n_kv_heads"] * a["head_dim"] * 2 * 2, rel=0.02)
