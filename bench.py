@@ -225,6 +225,27 @@ def run_reference(args, cfg):
     return 0
 
 
+# ---------------------------------------------------------------- replicas
+# One independent fingerprint per rank (the path does not shard): the ranks
+# exchange nothing but their timings.
+def rank_max(x, world, device):
+    """The largest of the ranks' values of x (the slowest rank's time)."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_tokens_per_s(world, batch, tokens_per_sequence, slowest_ms):
+    """Whole-job decode throughput: every rank decodes batch x tokens_per_sequence
+    tokens of its own replica, and the job takes as long as its slowest rank."""
+    return world * batch * tokens_per_sequence / (slowest_ms * 1e-3)
+
+
 def config_json(args, cfg):
     t, wq, kvq, B, S, N = cfg
     a = arch_dict(t)
@@ -350,11 +371,7 @@ def main():
             dist.barrier()
 
     def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return rank_max(x, world, "cuda")
 
     t, wq, kvq, B, S, N = cfg
     a = arch_dict(t)
@@ -383,7 +400,7 @@ def main():
         total_ms = max_over_ranks(sum(ttft) + sum(dec))
         dec_ms = max_over_ranks(sum(dec))
         ttft_ms = max_over_ranks(sum(ttft) / args.steps)
-        value = world * B * N * args.steps / (dec_ms * 1e-3)
+        value = replica_tokens_per_s(world, B, N * args.steps, dec_ms)
 
         # instrumented decode steps: per-block and per-kernel device time
         prof = fp.fp_profile(h, S, N, warmup=0, iters=1).as_dict()
@@ -401,7 +418,9 @@ def main():
         block_gbs = [bb / (bm * 1e-3) / 1e9 for bb, bm in zip(prof["block_bytes"], prof["block_ms"])]
         launches = args.steps * (prof["prefill_launches"] + N * prof["decode_launches"])
 
-        # end to end through the C ABI with host buffers
+        # end to end through the C ABI with host buffers: every decode step
+        # takes its input tokens from pinned host memory and returns the
+        # generated ones there (the prompt's prefill is set-up, as above)
         e2e = None
         if not args.no_e2e:
             pin_prompt = torch.empty((B, S), dtype=torch.int32, pin_memory=True)
@@ -409,22 +428,24 @@ def main():
             import synth
 
             host_prompt[:] = synth.tokens(0, B * S, a["vocab"]).reshape(B, S)
+            pin_in = torch.empty(B, dtype=torch.int32, pin_memory=True).numpy()
             pin_out = torch.empty(B, dtype=torch.int32, pin_memory=True).numpy()
-            fp.fp_prefill(h, host_prompt, out=pin_out)
-            for _ in range(N):
-                fp.fp_decode_step(h, None, out=pin_out)
-            barrier()
-            t_dec = 0.0
-            for _ in range(args.steps):
+
+            def host_request():
                 fp.fp_prefill(h, host_prompt, out=pin_out)
                 t0 = time.perf_counter()
                 for _ in range(N):
-                    fp.fp_decode_step(h, None, out=pin_out)
-                t_dec += time.perf_counter() - t0
+                    pin_in[:] = pin_out
+                    fp.fp_decode_step(h, pin_in, out=pin_out)
+                return time.perf_counter() - t0
+
+            host_request()
+            barrier()
+            t_dec = sum(host_request() for _ in range(args.steps))
             barrier()
             t_dec = max_over_ranks(t_dec)
-            e2e = {"value": world * B * N * args.steps / t_dec, "unit": "tokens/s",
-                   "h2d_bytes_per_step": B * S * 4, "d2h_bytes_per_step": B * 4 * (N + 1)}
+            e2e = {"value": replica_tokens_per_s(world, B, N * args.steps, 1e3 * t_dec), "unit": "tokens/s",
+                   "h2d_bytes_per_step": B * 4 * N, "d2h_bytes_per_step": B * 4 * N}
 
         cpu = None
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
