@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #define FP_DEV __device__ __forceinline__
 #define FP_HD __host__ __device__ __forceinline__
 
@@ -98,6 +100,22 @@ inline cudaError_t launch(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t 
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+// Lifts a kernel's dynamic shared-memory limit to `bytes` once per device:
+// function attributes belong to each device's context, so a process that
+// drives several GPUs sets it on each.  `done` (one per call site) holds a
+// bit per device ordinal below 64.
+template <typename... KArgs>
+inline cudaError_t smem_limit_once(void (*kern)(KArgs...), int bytes, std::atomic<unsigned long long>* done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if (done->load(std::memory_order_acquire) & bit) return cudaSuccess;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) done->fetch_or(bit, std::memory_order_acq_rel);
+  return e;
 }
 
 // SplitMix64 finaliser (Steele, Lea and Flood, OOPSLA 2014).  The generator's

@@ -471,12 +471,8 @@ bool attention_prefill_tc_ok(int B, int S, int n_heads, const fp_kv_view& kv, co
 template <bool KV8>
 static cudaError_t launch_pa_tc(const CUtensorMap& mq, const CUtensorMap& mk, const CUtensorMap& mv, int B, int S,
                                 int n_heads, const fp_kv_view& kv, uint16_t* out, int32_t* err, cudaStream_t s) {
-  static bool attr = false;
-  if (!attr) {
-    FP_CUDA_TRY(
-        cudaFuncSetAttribute(attn_prefill_tc_kernel<KV8>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPaSmem));
-    attr = true;
-  }
+  static std::atomic<unsigned long long> attr{0};
+  FP_CUDA_TRY(smem_limit_once(attn_prefill_tc_kernel<KV8>, kPaSmem, &attr));
   const dim3 grid((S + kPaB - 1) / kPaB, n_heads, B);
   return launch(attn_prefill_tc_kernel<KV8>, grid, dim3(pa_threads<KV8>()), (size_t)kPaSmem, s, mq, mk, mv,
                 (const int8_t*)kv.k_pool, (const int8_t*)kv.v_pool, (const float*)kv.k_scale,

@@ -332,11 +332,8 @@ static cudaError_t launch_tc_t(const CUtensorMap& mx, const CUtensorMap& mw, int
                                const uint16_t* scales, const uint16_t* R, void* Y, int32_t* err, cudaStream_t s) {
   auto kern = gemm_tc_kernel<EPI, SCALE>;
   const size_t smem = (size_t)kTcStages * kTcStageBytes + 1024;
-  static bool attr = false;
-  if (!attr) {
-    FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-    attr = true;
-  }
+  static std::atomic<unsigned long long> attr{0};
+  FP_CUDA_TRY(smem_limit_once(kern, (int)smem, &attr));
   const int Nout = EPI == FP_EPI_SWIGLU ? N / 2 : N;
   const int bn = kTcBN / (EPI == FP_EPI_SWIGLU ? 2 : 1);
   const long long tiles = (long long)((Nout + bn - 1) / bn) * ((M + kTcBM - 1) / kTcBM);

@@ -469,11 +469,8 @@ static cudaError_t launch_q4_t(const uint8_t* codes, const CUtensorMap& mx, int 
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
   auto kern = gemv_q4tc_kernel<MT, EPI>;
   const int smem = std::max(Q4Geom<MT, NR>::kSmem, kQ4MinSmem);
-  static bool attr = false;
-  if (!attr) {
-    FP_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    attr = true;
-  }
+  static std::atomic<unsigned long long> attr{0};
+  FP_CUDA_TRY(smem_limit_once(kern, smem, &attr));
   const int nout = NR == 2 ? N / 2 : N;
   const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
   const int S = K / 128;
