@@ -58,9 +58,11 @@ enum {
  * Kernel choice depends on M, N and K: M <= 64 runs the decode GEMV (the
  * work is cut into equal ranges of (128-row block, K step), one per resident
  * CTA, and shared blocks are reduced from fp32 partials in a fixed order) --
- * on the CUDA cores, except int4 with 17 <= M <= 64 and 16-byte aligned x and
- * codes, which runs on tcgen05 with each weight expanded to bf16((q - z) s)
- * as the prefill GEMM does -- larger M the tcgen05 GEMM.  workspace: 16-byte aligned, at least
+ * on mma.sync with the codes dequantised in registers, except int4 with
+ * 17 <= M <= 64 and 16-byte aligned x and codes, which runs on tcgen05 with
+ * each weight expanded to bf16((q - z) s) as the prefill GEMM does; a K that
+ * is not a multiple of the GEMV's K step falls back to one warp per output
+ * row on the CUDA cores -- larger M the tcgen05 GEMM.  workspace: 16-byte aligned, at least
  * fp_op_linear_workspace_bytes(wquant, M, N, K) bytes (may be NULL when that
  * is 0), else FP_ERR_INVALID_ARG.  Its leading bytes are ticket counters
  * that must be zero before the first call (e.g. a zeroed buffer); every call
