@@ -86,6 +86,24 @@ def test_op_argument_checks_on_host(fp):
     assert fp.fp_strerror(-5) == "KV cache capacity exceeded"
 
 
+def test_empty_inputs_are_no_ops(fp):
+    """Zero rows, sequences or tokens: every op returns success without
+    launching anything (this runs with no GPU at all)."""
+    import ctypes
+
+    L = fp._lib
+    kv = fp.fp_kv_view(0, 2, 128, 16, 4, 8, 1, 1, None, None, 1)
+    assert L.fp_op_attention_prefill(1, 1024, 0, 4, 4, ctypes.byref(kv), 1, None, None) == 0  # B = 0
+    assert L.fp_op_attention_prefill(1, 1024, 2, 0, 4, ctypes.byref(kv), 1, None, None) == 0  # S = 0
+    assert L.fp_op_attention_decode(1, 1024, 0, 4, ctypes.byref(kv), 1, 64, 1, None, 0, None, None) == 0
+    assert L.fp_op_rope_kv(1, 0, 4, 1536, 4, ctypes.byref(kv), 1, 1, None, None) == 0
+    assert L.fp_op_linear(1, 0, 1, 0, 128, 128, 1, 1, None, None, 1, None, 0, None) == 0
+    assert L.fp_op_rmsnorm(1, 0, 128, 128, 0, 1, ctypes.c_float(1e-5), 1, None) == 0
+    assert L.fp_op_embed(1, 0, 1, 32000, 128, 1, None, None) == 0
+    assert L.fp_op_argmax(1, 0, 32000, 1, None) == 0
+    assert L.fp_op_quantize(1, 1, 0, 128, 1, 1, None, None) == 0
+
+
 def test_forward_kernels_wait_for_their_predecessor():
     """Kernels of the forward pass are launched with programmatic dependent
     launch, so each must execute pdl_wait() before it reads or writes
