@@ -104,6 +104,28 @@ def test_empty_inputs_are_no_ops(fp):
     assert L.fp_op_quantize(1, 1, 0, 128, 1, 1, None, None) == 0
 
 
+def test_kernels_have_no_unbounded_waits_or_traps():
+    """Static check of the CUDA sources: no kernel can hang or trap the GPU
+    by construction.  mbarrier polling lives only in the bounded helpers of
+    tc.cuh (a fixed number of try_wait rounds, then the caller records an
+    error and leaves); there are no open-ended loops, no __trap() and no
+    device-side assert()."""
+    csrc = os.path.join(ROOT, "paper_2501_13111_gb300", "csrc")
+    bad = []
+    for name in sorted(os.listdir(csrc)):
+        if not name.endswith((".cu", ".cuh")):
+            continue
+        src = open(os.path.join(csrc, name)).read()
+        for pat in (r"while\s*\(\s*(true|1)\s*\)", r"for\s*\(\s*;\s*;\s*\)", r"__trap\s*\(", r"(?<![\w_])assert\s*\("):
+            for m in re.finditer(pat, src):
+                bad.append((name, src[: m.start()].count("\n") + 1, m.group(0)))
+        if name != "tc.cuh" and "try_wait" in src:
+            bad.append((name, 0, "mbarrier try_wait outside the bounded helpers"))
+    assert not bad, bad
+    tc = open(os.path.join(csrc, "tc.cuh")).read()
+    assert "kTcSpinLimit" in tc and tc.count("for (long long it = 0; it < kTcSpinLimit; ++it)") == tc.count("mbarrier.try_wait")
+
+
 def test_forward_kernels_wait_for_their_predecessor():
     """Kernels of the forward pass are launched with programmatic dependent
     launch, so each must execute pdl_wait() before it reads or writes
