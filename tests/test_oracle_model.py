@@ -201,3 +201,85 @@ def test_store_kv_modes():
     r8 = M.store_kv(x, M.KV_INT8)
     s = np.abs(r).max(axis=-1, keepdims=True) / 127
     assert np.all(np.abs(r8 - r) <= s / 2 * (1 + 1e-6))
+
+
+# ---------------------------------------------------------------- a whole block, brute force
+def _bf16_scalar(x):
+    """fp64 -> fp32 -> bf16, round to nearest even, on one scalar (bit arithmetic)."""
+    import struct
+
+    b = struct.unpack("<I", struct.pack("<f", float(np.float32(x))))[0]
+    b = (b + 0x7FFF + ((b >> 16) & 1)) >> 16
+    return struct.unpack("<f", struct.pack("<I", (b << 16) & 0xFFFFFFFF))[0]
+
+
+def _block_by_loops(a, w, h):
+    """One decoder block over h [T][d] at positions 0 .. T-1, every sum an
+    explicit scalar loop from the definitions (pre-norm RMSNorm, fused
+    [q | k | v] rows, rotate-half RoPE on q and k, bf16-rounded cache,
+    causal GQA softmax attention, O projection, SwiGLU over [gate | up]
+    rows, down projection, two residual adds)."""
+    import math
+
+    T, d = len(h), a.hidden
+    H, G, hd, f = a.n_heads, a.n_kv_heads, a.head_dim, a.ffn
+
+    def rms(x, g):
+        ms = sum(v * v for v in x) / len(x)
+        return [x[i] / math.sqrt(ms + a.rms_eps) * g[i] for i in range(len(x))]
+
+    def mat_row(W, r, x):
+        return sum(W[r][k] * x[k] for k in range(len(x)))
+
+    def rot(x, p):
+        out = list(x)
+        for i in range(hd // 2):
+            th = p * a.rope_base ** (-2.0 * i / hd)
+            c, s = math.cos(th), math.sin(th)
+            out[i] = x[i] * c - x[i + hd // 2] * s
+            out[i + hd // 2] = x[i + hd // 2] * c + x[i] * s
+        return out
+
+    Wqkv, Wo, Wgu, Wd = w[(0, "wqkv")], w[(0, "wo")], w[(0, "wgu")], w[(0, "wdown")]
+    q, k, v = [], [], []
+    for t in range(T):
+        y = rms(h[t], w[(0, "attn_norm")])
+        q.append([rot([mat_row(Wqkv, j * hd + i, y) for i in range(hd)], t) for j in range(H)])
+        k.append([[_bf16_scalar(e) for e in rot([mat_row(Wqkv, H * hd + j * hd + i, y) for i in range(hd)], t)]
+                  for j in range(G)])
+        v.append([[_bf16_scalar(mat_row(Wqkv, (H + G) * hd + j * hd + i, y)) for i in range(hd)] for j in range(G)])
+    out = []
+    for t in range(T):
+        o = []
+        for j in range(H):
+            kv = j // (H // G)
+            sc = [sum(q[t][j][i] * k[u][kv][i] for i in range(hd)) / math.sqrt(hd) for u in range(t + 1)]
+            m = max(sc)
+            e = [math.exp(s - m) for s in sc]
+            z = sum(e)
+            o += [sum(e[u] / z * v[u][kv][i] for u in range(t + 1)) for i in range(hd)]
+        h1 = [h[t][r] + mat_row(Wo, r, o) for r in range(d)]
+        y2 = rms(h1, w[(0, "ffn_norm")])
+        act = []
+        for c in range(f):
+            gt, up = mat_row(Wgu, c, y2), mat_row(Wgu, f + c, y2)
+            act.append(gt / (1.0 + math.exp(-gt)) * up)
+        out.append([h1[r] + mat_row(Wd, r, act) for r in range(d)])
+    return out
+
+
+def test_block_matches_brute_force_loops():
+    """The oracle's vectorised block against the same block written out as
+    scalar loops on a tiny GQA shape (H 4, Hkv 2, hd 4, d 8, f 6, T 5): a
+    transposed weight, a wrong q/k/v or gate/up row range, RoPE on v or a
+    wrong head mapping all change the result by O(1)."""
+    rng = np.random.default_rng(11)
+    a = M.Arch(n_layers=1, hidden=8, n_heads=4, n_kv_heads=2, head_dim=4, ffn=6, vocab=7, rms_eps=1e-5)
+    w = {(0, "attn_norm"): rng.uniform(0.5, 1.5, 8), (0, "ffn_norm"): rng.uniform(0.5, 1.5, 8),
+         (0, "wqkv"): rng.normal(0, 0.5, ((4 + 2 * 2) * 4, 8)), (0, "wo"): rng.normal(0, 0.5, (8, 16)),
+         (0, "wgu"): rng.normal(0, 0.5, (12, 8)), (0, "wdown"): rng.normal(0, 0.5, (8, 6))}
+    h = rng.normal(0, 1, (5, 8))
+    fp = M.Fingerprint(a, w, M.KV_BF16, 1, 8)
+    got = fp._block(0, h[None], 0)[0]
+    ref = np.array(_block_by_loops(a, w, h.tolist()))
+    assert np.allclose(got, ref, rtol=1e-10, atol=1e-12), np.max(np.abs(got - ref))
