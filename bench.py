@@ -118,18 +118,59 @@ CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active
 
 
 class ClockSampler:
+    """nvidia-smi sampling SM clocks and throttle reasons every 25 ms.  The
+    timed region starts only once the first sample has arrived (so the
+    samples that follow fall inside it); that first sample is kept apart and
+    reported only when the region ended before the next one."""
+
+    PERIOD_MS = 25
+
     def __init__(self, index):
         self.index = index
         self.proc = None
+        self.first = []
+        self.lines = []
 
     def __enter__(self):
+        for period in (self.PERIOD_MS, 200):  # 200 ms if this nvidia-smi refuses the shorter period
+            if self._start(period) != "refused":
+                break
+        return self
+
+    def _start(self, period):
+        import select
+
+        self.first = []
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={CLOCK_Q}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", str(period)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
-        return self
+            return "absent"
+        # wait (at most 5 s) for the sampler's first line, reading the raw pipe
+        # so that communicate() later sees every byte that follows
+        fd, buf, eof = self.proc.stdout.fileno(), b"", False
+        deadline = time.time() + 5.0
+        while b"\n" not in buf:
+            left = deadline - time.time()
+            if left <= 0 or not select.select([fd], [], [], left)[0]:
+                break
+            chunk = os.read(fd, 4096)
+            if not chunk:
+                eof = True
+                break
+            buf += chunk
+        self.first = [l for l in buf.decode(errors="replace").splitlines() if l.strip()]
+        if not self.first and eof:  # it closed its output without a sample: it refused the arguments
+            try:
+                self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.proc.communicate()
+            self.proc = None
+            return "refused"
+        return "ok"
 
     def __exit__(self, *exc):
         self.lines = []
@@ -140,7 +181,7 @@ class ClockSampler:
             except subprocess.TimeoutExpired:
                 self.proc.kill()
                 out, _ = self.proc.communicate()
-            self.lines = [l for l in out.splitlines() if l.strip()]
+            self.lines = [l for l in out.splitlines() if l.strip()] or self.first
         return False
 
     def summary(self):

@@ -56,3 +56,39 @@ def test_kernel_bytes_closed_forms():
     assert kb["lm_head"] == 2 * V * d + 2 * B * d + 4 * B * V
     # one block's K and V: B x context x Hkv x hd x 2 (K and V) x 2 bytes
     assert kb["attn"] == pytest.approx(B * S * a["n_kv_heads"] * a["head_dim"] * 2 * 2, rel=0.02)
+
+
+FAKE_SMI = """#!/bin/bash
+# stands in for nvidia-smi: refuses sampling periods below MIN_MS, else prints
+# one CSV sample per period (SM MHz counting up from 2000) until killed
+for a in "$@"; do last=$a; done
+if [ "$last" -lt {min_ms} ]; then echo "Invalid value" >&2; exit 2; fi
+sleep 0.2
+i=0
+while true; do
+  echo "0, $((2000 + i)), 2070, 900.00, 0x0, Not Active, Not Active, Not Active, {cap}"
+  i=$((i+1)); sleep 0.02
+done
+"""
+
+
+@pytest.mark.parametrize("min_ms,cap", [(1, "Active"), (100, "Not Active")])
+def test_clock_sampler_samples_inside_the_region(tmp_path, monkeypatch, min_ms, cap):
+    """The sampler waits for nvidia-smi's first sample before the timed
+    region starts, keeps the samples taken inside it, falls back to a 200 ms
+    period when the short one is refused, and reports the power cap."""
+    import time
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    smi = tmp_path / "nvidia-smi"
+    smi.write_text(FAKE_SMI.format(min_ms=min_ms, cap=cap))
+    smi.chmod(0o755)
+    monkeypatch.setenv("PATH", f"{tmp_path}:{os.environ['PATH']}")
+    with bench.ClockSampler(0) as c:
+        time.sleep(0.5)
+    s = c.summary()
+    assert s["sm_max_mhz"] == 2070.0 and s["samples"] >= 2
+    assert all(line.split(",")[1].strip() != "2000" for line in c.lines)  # the pre-region sample is left out
+    assert s["reasons"] == (["sw_power_cap"] if cap == "Active" else [])
