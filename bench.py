@@ -425,9 +425,9 @@ def main():
             fp.fp_decode_steps(h, N)
         torch.cuda.synchronize()
         ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-        barrier()
-        torch.cuda.synchronize()
-        with ClockSampler(local) as clk:
+        with ClockSampler(local) as clk:  # sampling before the barrier, so every rank's region starts together
+            barrier()
+            torch.cuda.synchronize()
             for k in range(args.steps):
                 ev[k][0].record(stream)
                 fp.fp_prefill(h, None, want_next=False, prompt_len=S)
