@@ -126,6 +126,43 @@ def test_kernels_have_no_unbounded_waits_or_traps():
     assert "kTcSpinLimit" in tc and tc.count("for (long long it = 0; it < kTcSpinLimit; ++it)") == tc.count("mbarrier.try_wait")
 
 
+def test_binding_struct_layouts_match_the_headers(fp, tmp_path):
+    """The ctypes mirrors of the ABI structs have the C compiler's sizes and
+    field offsets (a C program built against include/*.h prints them)."""
+    import ctypes
+    import shutil
+    import subprocess
+
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    structs = [fp.fp_arch, fp.fp_allocator, fp.fp_profile_result, fp.fp_plan, fp.fp_kv_view, fp.fp_eq1_fit,
+               fp.fp_l2_terms]
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "fp.h"', '#include "fp_ops.h"',
+             '#include "fp_estimate.h"', "int main(void) {"]
+    for st in structs:
+        n = st.__name__
+        lines.append(f'  printf("{n} sizeof %zu\\n", sizeof({n}));')
+        for fname, _ in st._fields_:
+            lines.append(f'  printf("{n} {fname} %zu\\n", offsetof({n}, {fname}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split("\n")
+    want = {}
+    for line in out:
+        if line.strip():
+            name, field, val = line.split()
+            want[(name, field)] = int(val)
+    for st in structs:
+        n = st.__name__
+        assert want[(n, "sizeof")] == ctypes.sizeof(st), n
+        for fname, _ in st._fields_:
+            assert want[(n, fname)] == getattr(st, fname).offset, (n, fname)
+
+
 def test_forward_kernels_wait_for_their_predecessor():
     """Kernels of the forward pass are launched with programmatic dependent
     launch, so each must execute pdl_wait() before it reads or writes
