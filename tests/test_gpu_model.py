@@ -198,6 +198,7 @@ def test_profile_reports(fp):
         assert r.ttft_ms > 0 and r.tpot_ms > 0 and r.decode_tokens_per_s > 0
         assert r.weight_bytes == memory.weight_bytes(arch, 1)
         assert r.decode_bytes_per_step == int(memory.decode_step_bytes(arch, 1, 0, 4, 64 + 8.5))
+        assert r.prefill_flops == memory.prefill_flops(arch, 4, 64)
         assert all(x > 0 for x in list(r.block_ms)[:2])
         # embed + first norm; per block 7 launches (6 in the first) + decode attention (1, or 2 with a
         # combine pass); final norm, head, argmax (which also advances the positions)

@@ -58,3 +58,51 @@ def test_memory_extrapolation_linear():
     per, base = 1.25e9, 3.0e9
     m = estimator.extrapolate_memory(1, base + per, 2, base + 2 * per, 80)
     assert m == base + 80 * per
+
+
+# ---------------------------------------------------------------- prefill FLOPs
+def _golden(name):
+    import json
+    import os
+
+    return json.load(open(os.path.join(os.path.dirname(__file__), "golden", name)))
+
+
+def test_prefill_flops_hand_counted_example():
+    g = _golden("prefill_flops_example.json")
+    a = Arch(**g["arch"])
+    assert memory.prefill_flops(a, g["batch"], g["prompt"]) == g["total"]
+
+
+def _loop_count_macs(arch, B, S):
+    """Multiply-adds of a prefill, counted by walking the forward pass with
+    explicit loops: each output element of a linear costs K multiply-adds,
+    each causal (query, key) pair hd for the score and hd for the value
+    product, the LM head one row of the last position per sequence."""
+    lin = att_pairs = head = 0
+    d, f, hd = arch.hidden, arch.ffn, arch.head_dim
+    for _ in range(arch.n_layers):
+        for _b in range(B):
+            for _s in range(S):
+                for n_out, k in ((arch.q_dim + 2 * arch.kv_dim, d), (d, arch.q_dim), (2 * f, d), (d, f)):
+                    lin += n_out * k
+            for _h in range(arch.n_heads):
+                for i in range(S):
+                    for _j in range(i + 1):
+                        att_pairs += 1
+    for _b in range(B):
+        head += arch.vocab * d
+    return lin, att_pairs * 2 * hd, head
+
+
+@pytest.mark.parametrize("shape", [(1, 4, 2, 1, 2, 3, 5, 2, 3), (2, 64, 4, 2, 16, 96, 50, 3, 7),
+                                   (1, 32, 8, 8, 4, 40, 11, 1, 1)])
+def test_prefill_flops_against_loop_count(shape):
+    *arch_t, B, S = shape
+    a = Arch(*arch_t)
+    lin, att, head = _loop_count_macs(a, B, S)
+    # the closed form counts S^2/2 (query, key) pairs per head where the loops
+    # count S(S+1)/2: S/2 pairs fewer, 2 hd multiply-adds each, per head,
+    # sequence and layer
+    fewer = a.n_layers * B * a.n_heads * S * a.head_dim
+    assert memory.prefill_flops(a, B, S) == 2 * (lin + att - fewer + head)
