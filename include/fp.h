@@ -146,6 +146,8 @@ int fp_load_prompt(fp_handle* h, const int32_t* host_tokens, int prompt_len);
 
 /* Prefill: run the prompt through the fingerprint from an empty cache, fill
  * the KV cache and emit the first generated token per sequence (greedy).
+ * This is the dummy request of the profiling step (Sec. 4.2, step 1) up to
+ * its first token: its duration is the TTFT of Eq. 1 (Sec. 5.3).
  * host_tokens [batch][prompt_len] is uploaded first; with host_tokens NULL
  * the resident prompt of fp_load_prompt is used (prompt_len must equal its
  * length, else FP_ERR_STATE).  host_next [batch] or NULL; with NULL the
@@ -154,7 +156,9 @@ int fp_prefill(fp_handle* h, const int32_t* host_tokens, int prompt_len, int32_t
 
 /* One decode step: consume one token per sequence (host_in [batch], or NULL
  * for the previous step's outputs kept on the device), append one position,
- * emit the next greedy token (host_out [batch] or NULL).  FP_ERR_STATE
+ * emit the next greedy token (host_out [batch] or NULL).  One step is one
+ * output token of Eq. 1 (Sec. 5.3); the KV cache makes every step cost the
+ * same work per layer (the passage before Eq. 1), so its duration is TPOT.  FP_ERR_STATE
  * before any prefill; FP_ERR_CAPACITY when the cache is full.  The step is a
  * replayed CUDA graph (captured on first use). */
 int fp_decode_step(fp_handle* h, const int32_t* host_in, int32_t* host_out);
@@ -195,7 +199,12 @@ typedef struct fp_profile_result {
                                  events, mean over iters (the latency of Eq. 1) */
 } fp_profile_result;
 
-/* Profile latency and memory: `warmup` untimed passes, then `iters` timed
+/* Profile latency and memory, the observations the estimator consumes:
+ * TTFT and TPOT of Eq. 1 (Sec. 5.3; with two fingerprint depths, Eqs. 2-3
+ * separate their per-layer and other parts) and the footprint W + A of the
+ * memory model (Sec. 5.2, TP = PP = 1), as the profiling step reads them
+ * from a deployed fingerprint (Sec. 4.2, step 1; Sec. 7 "Monitoring
+ * Daemon").  `warmup` untimed passes, then `iters` timed
  * passes of prefill(prompt_len) + n_decode decode steps on the batch;
  * prompt = host_prompt [batch][prompt_len] or, if NULL, SplitMix64 token ids
  * drawn from the handle's seed.  prompt_len + n_decode <= max_context. */
@@ -223,6 +232,13 @@ enum {
   FP_G_LENGTH = 11   /* int32 [batch] cached positions per sequence              */
 };
 long long fp_get_tensor(fp_handle* h, int what, int layer, int mat, void* host_dst, size_t bytes);
+
+/* As fp_get_tensor, from byte `offset` of the tensor on: returns the bytes
+ * written, or (host_dst NULL) the bytes from offset to the end; an offset
+ * past the end is FP_ERR_INVALID_ARG.  Lets a test read one sequence's rows
+ * of FP_G_HIDDEN (sequence b starts at b * rows_per_sequence * d * 2). */
+long long fp_get_tensor_at(fp_handle* h, int what, int layer, int mat, size_t offset, void* host_dst,
+                           size_t bytes);
 
 /* Byte plan of the handle (what fp_profile reports as peak_hbm_bytes). */
 typedef struct fp_plan {

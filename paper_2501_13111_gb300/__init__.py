@@ -126,6 +126,7 @@ _PROTOS = {
     "fp_decode_step": (_I, [_P, _P, _P]),
     "fp_profile": (_I, [_P, _I, _I, _I, _I, _P, C.POINTER(fp_profile_result)]),
     "fp_get_tensor": (_LL, [_P, _I, _I, _I, _P, _SZ]),
+    "fp_get_tensor_at": (_LL, [_P, _I, _I, _I, _SZ, _P, _SZ]),
     "fp_get_plan": (_I, [_P, C.POINTER(fp_plan)]),
     "fp_last_error": (C.c_char_p, [_P]),
     "fp_strerror": (C.c_char_p, [_I]),
@@ -140,6 +141,7 @@ _PROTOS = {
     "fp_op_rope_kv": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P, _P]),
     "fp_op_attention_decode": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _SZ, _P, _P]),
     "fp_op_attention_decode_workspace_bytes": (_SZ, [_I, _I, _I, _I]),
+    "fp_op_attention_decode_splits": (_I, [_I, _I, _I]),
     "fp_op_attention_decode_noalloc": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _P]),
     "fp_op_attention_prefill": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P]),
     "fp_op_argmax": (_I, [_P, _I, _I, _P, _P]),
@@ -240,15 +242,16 @@ def fp_profile(h, prompt_len, n_decode, warmup=1, iters=3, prompt=None):
     return res
 
 
-def fp_get_tensor(h, what, layer=0, mat=0, dtype=None, count=None):
+def fp_get_tensor(h, what, layer=0, mat=0, dtype=None, count=None, offset=0):
     """With dtype None returns the byte size, else a host array of that dtype
-    (its first ``count`` elements when given)."""
-    n = _check(_lib.fp_get_tensor(h, what, layer, mat, None, 0), h)
+    (its first ``count`` elements when given, from element ``offset`` on)."""
     if dtype is None:
-        return n
-    k = n // np.dtype(dtype).itemsize
+        return _check(_lib.fp_get_tensor(h, what, layer, mat, None, 0), h)
+    isz = np.dtype(dtype).itemsize
+    n = _check(_lib.fp_get_tensor_at(h, what, layer, mat, offset * isz, None, 0), h)
+    k = n // isz
     buf = np.empty(k if count is None else min(k, count), dtype=dtype)
-    _check(_lib.fp_get_tensor(h, what, layer, mat, _ptr(buf), buf.nbytes), h)
+    _check(_lib.fp_get_tensor_at(h, what, layer, mat, offset * isz, _ptr(buf), buf.nbytes), h)
     return buf
 
 
@@ -315,7 +318,11 @@ def fp_op_attention_decode(q, q_stride, B, n_heads, kv: fp_kv_view, lens, max_le
                                               workspace_bytes, err, stream))
 
 
-FP_NOALLOC_SCRATCH_BYTES = 32 << 20
+def fp_op_attention_decode_splits(B, n_kv_heads, max_len):
+    return _lib.fp_op_attention_decode_splits(B, n_kv_heads, max_len)
+
+
+FP_NOALLOC_SCRATCH_BYTES = 32 << 20  # FP_NOALLOC_SCRATCH_BYTES of fp_ops.h (a CPU test keeps the two equal)
 
 
 def fp_op_attention_decode_noalloc(q, q_stride, B, n_heads, kv: fp_kv_view, lens, max_len, out, err=None,

@@ -719,6 +719,10 @@ int fp_decode_step(fp_handle* h, const int32_t* host_in, int32_t* host_out) {
 }
 
 long long fp_get_tensor(fp_handle* h, int what, int layer, int mat, void* host_dst, size_t bytes) {
+  return fp_get_tensor_at(h, what, layer, mat, 0, host_dst, bytes);
+}
+
+long long fp_get_tensor_at(fp_handle* h, int what, int layer, int mat, size_t offset, void* host_dst, size_t bytes) {
   if (!h) return FP_ERR_INVALID_ARG;
   const void* src = nullptr;
   size_t n = 0;
@@ -752,11 +756,12 @@ long long fp_get_tensor(fp_handle* h, int what, int layer, int mat, void* host_d
     case FP_G_LENGTH: src = h->pos; n = (size_t)h->B * 4; break;
     default: return h->fail(FP_ERR_INVALID_ARG, "unknown tensor");
   }
-  if (!host_dst) return (long long)n;
-  n = std::min(n, bytes);  // a smaller buffer receives the leading bytes
+  if (offset > n) return h->fail(FP_ERR_INVALID_ARG, "offset past the end of the tensor");
+  if (!host_dst) return (long long)(n - offset);
+  n = std::min(n - offset, bytes);  // a smaller buffer receives the leading bytes from offset on
   if (n == 0) return 0;
   cudaError_t e = cudaStreamSynchronize(h->stream);
-  if (e == cudaSuccess) e = cudaMemcpy(host_dst, src, n, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(host_dst, (const char*)src + offset, n, cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return h->cuda_fail(e, "get tensor");
   return (long long)n;
 }

@@ -1,7 +1,9 @@
 """Parity at the full sizes of the workloads, in the launch configuration the
 bench times.
 
-* Llama-2-7B- and 13B-shaped fingerprints end to end: the handle is created
+* Llama-2-7B-, 13B- and 70B-shaped fingerprints end to end (the 70B shape:
+  int4 g128 weights, int8 KV cache, GQA 64/8, batch 32, 2048-token prompts,
+  the bench's default workload): the handle is created
   exactly as ``bench.py`` creates it (device-side seeded weights, seed 0, unit
   norm gains, the full batch, prompt and context), prefills the full batch and
   decodes a few steps.  The oracle runs a batch-1 slice per checked sequence
@@ -10,7 +12,7 @@ bench times.
   ids are compared (tolerance and near-tie rule as in test_gpu_model).  The
   decode steps feed the oracle's token to the checked sequences and the
   device's own token to the others.
-* Llama-2-70B-shaped: the kernels at the workload's full shapes, through the
+* Llama-2-70B-shaped, op level as well: the kernels at the workload's full shapes, through the
   op entry points (same kernels and plans as the runtime): the four int4
   decode linears and the LM head at M = 32 on sampled output rows, the GQA
   int8-KV decode attention at B 32 and context 2148 on sampled (sequence,
@@ -32,6 +34,8 @@ FULL = {
     # name: (arch, wquant, kvquant, batch, prompt, decode steps of the bench, checked sequences)
     "l7b": (M.Arch(2, 4096, 32, 32, 128, 11008, 32000), 1, 0, 8, 512, 100, [0, 7]),
     "l13b": (M.Arch(2, 5120, 40, 40, 128, 13824, 32000), 2, 0, 16, 1024, 100, [5]),
+    # the first and the last sequence: rows at both ends of M = 65536 in prefill
+    "l70b": (M.Arch(2, 8192, 64, 8, 128, 28672, 32000), 2, 1, 32, 2048, 100, [0, 31]),
 }
 N_CHECKED_DECODE = 3
 
@@ -44,18 +48,34 @@ def fp():
     return fp
 
 
-def _near_tie_ok(got, ref_logits, tau):
+# int8 KV cache, end to end: the device and the oracle each quantise K and V
+# per (token, head) from bf16 values that differ by one rounding, which flips
+# codes by one step (about one in six); the 70B-shaped synthetic attention is
+# sharp (scores with a standard deviation of about 3), and two blocks amplify
+# the flips and the bf16 storage of activations to about 5 % of the logits'
+# range (measured: 4.7 % and 5.1 % on the first and last sequence, while each
+# block alone with the oracle's codes stays at about 1 %:
+# test_full_size_70b_blocks_with_the_oracles_kv_codes).  End-to-end
+# comparisons with an int8 cache are held to 1e-1; the kernels' own error is
+# held to 2e-2 by that test.
+TAU_E2E_KV8 = 1e-1
+
+
+def _near_tie_ok(got, ref_logits, dev_logits):
+    """A greedy id may differ from the oracle's only where the measured logit
+    error could reorder the oracle's top two (their gap below twice the
+    largest |device - oracle| logit difference of that row)."""
     ref = int(M.argmax(ref_logits[None])[0])
     if got == ref:
         return True
     top = np.sort(ref_logits)[-2:]
-    return top[1] - top[0] < 2 * tau * np.max(np.abs(ref_logits))
+    return top[1] - top[0] < 2 * np.max(np.abs(np.asarray(dev_logits, np.float64) - ref_logits))
 
 
 @pytest.mark.parametrize("name", list(FULL))
 def test_full_size_sequences_match_oracle(fp, name):
     arch, wq, kvq, B, S, N, seqs = FULL[name]
-    tau = TAU[wq]
+    tau = TAU_E2E_KV8 if kvq == 1 else TAU[wq]
     T = S + N + 1  # the bench's context
     get = weight_getter(0, gains="ones")  # the bench's device-side init: seed 0, unit gains
     with ThreadPoolExecutor(max_workers=8) as pool:
@@ -75,34 +95,37 @@ def test_full_size_sequences_match_oracle(fp, name):
                                           p["zeros"].reshape(-1))
         toks = synth.tokens(0, B * S, arch.vocab).reshape(B, S)
         nxt = fp.fp_prefill(h, toks)
-        hid = [quant.bf16_to_f32(fp.fp_get_tensor(h, fp.FP_G_HIDDEN, l, 0, np.uint16)).reshape(B, S, arch.hidden)
-               for l in range(arch.n_layers)]
+        d = arch.hidden
+
+        def seq_hidden(l, b, rows):
+            """Block l's output rows of sequence b (rows per sequence), read alone."""
+            bits = fp.fp_get_tensor(h, fp.FP_G_HIDDEN, l, 0, np.uint16, count=rows * d, offset=b * rows * d)
+            return quant.bf16_to_f32(bits).reshape(rows, d)
+
         lg = fp.fp_get_tensor(h, fp.FP_G_LOGITS, 0, 0, np.float32).reshape(B, arch.vocab)
         refs = {b: M.Fingerprint(arch, w, kvq, 1, T) for b in seqs}
         cur = nxt.copy()
         for b in seqs:
             out = refs[b].prefill(toks[b:b + 1])
             for l in range(arch.n_layers):
-                e = rel_err(hid[l][b], out["hidden"][l][0])
+                e = rel_err(seq_hidden(l, b, S), out["hidden"][l][0])
                 assert e <= tau, (name, "prefill hidden", b, l, e)
             e = rel_err(lg[b], out["logits"][0])
             assert e <= tau, (name, "prefill logits", b, e)
-            assert _near_tie_ok(int(nxt[b]), out["logits"][0], tau), (name, "prefill token", b)
+            assert _near_tie_ok(int(nxt[b]), out["logits"][0], lg[b]), (name, "prefill token", b)
             cur[b] = out["tokens"][0]
         for step in range(N_CHECKED_DECODE):
             got = fp.fp_decode_step(h, cur)
-            hid = [quant.bf16_to_f32(fp.fp_get_tensor(h, fp.FP_G_HIDDEN, l, 0, np.uint16)).reshape(B, arch.hidden)
-                   for l in range(arch.n_layers)]
             lg = fp.fp_get_tensor(h, fp.FP_G_LOGITS, 0, 0, np.float32).reshape(B, arch.vocab)
             nxt_cur = got.copy()
             for b in seqs:
                 out = refs[b].decode([cur[b]])
                 for l in range(arch.n_layers):
-                    e = rel_err(hid[l][b], out["hidden"][l][0])
+                    e = rel_err(seq_hidden(l, b, 1)[0], out["hidden"][l][0])
                     assert e <= tau, (name, "decode hidden", step, b, l, e)
                 e = rel_err(lg[b], out["logits"][0])
                 assert e <= tau, (name, "decode logits", step, b, e)
-                assert _near_tie_ok(int(got[b]), out["logits"][0], tau), (name, "decode token", step, b)
+                assert _near_tie_ok(int(got[b]), out["logits"][0], lg[b]), (name, "decode token", step, b)
                 nxt_cur[b] = out["tokens"][0]
             cur = nxt_cur
     finally:
@@ -213,3 +236,95 @@ def test_full_size_70b_prefill_gate_up(fp):
     yu = xf @ _oracle_rows(wq, stream, ncols + nout, k).T
     ref = M.silu(yg) * yu
     assert rel_err(got, ref) <= TAU[wq] / 4, rel_err(got, ref)
+
+
+def test_full_size_70b_blocks_with_the_oracles_kv_codes(fp):
+    """The kernels of the 70B-shaped workload, block by block, with the int8
+    KV reading taken out: one 2048-token sequence through the op entry points
+    (RMSNorm, the int4 prefill GEMMs, RoPE + int8 KV append, tcgen05 prefill
+    attention over the int8 cache, SwiGLU, residual adds, final norm, LM head)
+    where each block starts from the oracle's own input to that block and its
+    cache holds the oracle's K/V codes and scales, written over the ones the
+    device quantised.  Two independent int8 quantisations of K and V from bf16
+    values that differ by one rounding flip codes by one step, and sharp
+    attention amplifies that through the blocks (the end-to-end comparison
+    above); with the codes shared, what remains is the kernels' own error
+    (bf16 storage of activations, fp32 accumulation), held to 2e-2."""
+    torch = torch_mod()
+    a = A70
+    S, d, f, H, Hkv, hd = 2048, a.hidden, a.ffn, a.n_heads, a.n_kv_heads, a.head_dim
+    nqkv = a.q_dim + 2 * a.kv_dim
+    get = weight_getter(0, gains="ones")
+    with ThreadPoolExecutor(max_workers=8) as pool:
+        w, payload = M.build_weights(a, 2, get, map_fn=pool.map)
+    toks = synth.tokens(0, S, a.vocab).reshape(1, S)
+    # device weights: the oracle's codes, scales and zeros of every block matrix
+    mats = {}
+    for l in range(a.n_layers):
+        for name in ("wqkv", "wo", "wgu", "wdown"):
+            p = payload[(l, name)]
+            mats[(l, name)] = (dev(p["codes"]), dev(p["scales"]), dev(p["zeros"]))
+    ones = dev(synth.f32_to_bf16_bits(np.ones(d, np.float32)))
+    head = dev(get(-1, 2, (a.vocab, d)))
+    # a batch-1 paged int8 cache with the identity page table
+    pps = S // 16
+    kpool, vpool = empty(pps * Hkv * 16 * hd), empty(pps * Hkv * 16 * hd)
+    ksc, vsc = empty(pps * Hkv * 16, np.float32), empty(pps * Hkv * 16, np.float32)
+    table = dev(np.arange(pps, dtype=np.int32).reshape(1, pps))
+    kv = fp.fp_kv_view(1, Hkv, hd, 16, pps, pps, ptr(kpool), ptr(vpool), ptr(ksc), ptr(vsc), ptr(table))
+    cs = empty(pps * 16 * hd // 2 * 2, np.float32)
+    fp.fp_op_rope_table(pps * 16, hd, a.rope_base, ptr(cs))
+    pos = dev(np.zeros(1, np.int32))
+    err = empty(1, np.int32)
+    y, qkv = empty(S * d * 2), empty(S * nqkv * 2)
+    att, act = empty(S * a.q_dim * 2), empty(S * f * 2)
+    wsb = max(fp.fp_op_linear_workspace_bytes(2, S, n, k) for n, k in ((nqkv, d), (d, a.q_dim), (2 * f, d), (d, f)))
+    ws = empty(wsb)
+
+    def lin(epi, x, name, l, n, k, out, resid=None):
+        c, sc, z = mats[(l, name)]
+        fp.fp_op_linear(2, epi, ptr(x), S, n, k, ptr(c), ptr(sc), ptr(z), ptr(resid), ptr(out), ptr(ws), wsb)
+
+    h_in = w["embed"][toks]  # [1, S, d], exact bf16 values
+    for l in range(a.n_layers):
+        # the oracle's block l from h_in, recording the K and V it stores
+        seen = []
+        orig = M.store_kv
+        M.store_kv = lambda x, kvq: (seen.append(x), orig(x, kvq))[1]
+        try:
+            ref_out = M.Fingerprint(a, w, 1, 1, S)._block(l, h_in, 0)[0]
+        finally:
+            M.store_kv = orig
+        kc, ks = quant.quantize_kv_int8(quant.f32_to_bf16_rne(seen[0][0].astype(np.float32)))  # [S, Hkv, hd]
+        vc, vs = quant.quantize_kv_int8(quant.f32_to_bf16_rne(seen[1][0].astype(np.float32)))
+        # the device's block l from the same input
+        h = dev(synth.f32_to_bf16_bits(h_in[0].astype(np.float32)))
+        fp.fp_op_rmsnorm(ptr(h), S, d, 1, 0, ptr(ones), a.rms_eps, ptr(y))
+        lin(0, y, "wqkv", l, nqkv, d, qkv)
+        fp.fp_op_rope_kv(ptr(qkv), 1, S, nqkv, H, kv, ptr(pos), ptr(cs), ptr(err))
+        torch.cuda.synchronize()
+        page = lambda x: np.ascontiguousarray(x.reshape(pps, 16, Hkv, *x.shape[2:]).swapaxes(1, 2))
+        kpool.copy_(torch.from_numpy(page(kc).reshape(-1).view(np.uint8)))
+        vpool.copy_(torch.from_numpy(page(vc).reshape(-1).view(np.uint8)))
+        ksc.copy_(torch.from_numpy(page(ks).reshape(-1)))
+        vsc.copy_(torch.from_numpy(page(vs).reshape(-1)))
+        fp.fp_op_attention_prefill(ptr(qkv), nqkv, 1, S, H, kv, ptr(att), ptr(err))
+        lin(1, att, "wo", l, d, a.q_dim, h, resid=h)
+        fp.fp_op_rmsnorm(ptr(h), S, d, 1, 0, ptr(ones), a.rms_eps, ptr(y))
+        lin(2, y, "wgu", l, 2 * f, d, act)
+        lin(1, act, "wdown", l, d, f, h, resid=h)
+        got = quant.bf16_to_f32(host(h, np.uint16)).reshape(S, d)
+        e = rel_err(got, ref_out)
+        assert e <= 2e-2, ("block", l, e)
+        h_in = quant.bf16_to_f32(synth.f32_to_bf16_bits(ref_out.astype(np.float32))).astype(np.float64)[None]
+    # final norm and LM head on the oracle's last hidden row
+    last = dev(synth.f32_to_bf16_bits(h_in[0, -1:].astype(np.float32)))
+    yl = empty(d * 2)
+    fp.fp_op_rmsnorm(ptr(last), 1, d, 1, 0, ptr(ones), a.rms_eps, ptr(yl))
+    lg = empty(a.vocab * 4)
+    lws = fp.fp_op_linear_workspace_bytes(0, 1, a.vocab, d)
+    lw = empty(max(lws, 16))
+    fp.fp_op_linear(0, 3, ptr(yl), 1, a.vocab, d, ptr(head), None, None, None, ptr(lg), ptr(lw), lws)
+    ref_lg = M.rmsnorm(h_in[0, -1], w["final_norm"], a.rms_eps) @ w["lm_head"].T
+    assert rel_err(host(lg, np.float32), ref_lg) <= 2e-2
+    assert host(err, np.int32)[0] == 0

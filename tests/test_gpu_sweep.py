@@ -6,10 +6,14 @@ x KV cache {bf16, int8} x batch {1, 8, 32, 64} x context {128, 512, 2048,
 Every point runs the way the sweep measures it: fp_create with device-side
 seeded weights, a prefill of the full batch at the full context, then
 fp_profile with decode steps.  Each point is checked against the oracle on a
-batch-1 slice: sequence 0's first 64 positions after the block.  Attention is
-causal, so those rows do not depend on the rest of the prompt; their
-reference is computed once per (weights, KV) pair, from the oracle's own
-seeded weights and tokens.  Decode steps at these shapes are checked by
+batch-1 slice: every sequence's prompt opens with the same 64 tokens, and the
+first 64 positions after the block of the first AND the last sequence are
+compared -- the last sequence's rows sit at the end of the prefill's
+M = batch x context rows (the last tiles of the GEMMs' persistent schedule,
+the last (sequence, head) pairs of the attention).  Attention is causal, so
+those rows do not depend on the rest of the prompt; their reference is
+computed once per (weights, KV) pair, from the oracle's own seeded weights
+and tokens.  Decode steps at these shapes are checked by
 test_gpu_fullsize and test_gpu_model.
 """
 from concurrent.futures import ThreadPoolExecutor
@@ -70,14 +74,17 @@ def test_sweep_points_match_oracle(fp, raw_weights, wq, kvq):
     tau = max(TAU[wq], TAU_KV8) if kvq == 1 else TAU[wq]
     for B in BATCH:
         for ctx in CONTEXT:
-            toks = stream[: B * ctx].reshape(B, ctx)
+            toks = stream[: B * ctx].reshape(B, ctx).copy()
+            toks[:, :PREFIX] = stream[:PREFIX]  # the shared prefix the reference covers
             h = fp.fp_create(arch_dict(a), wq, kvq, B, ctx + 100 + 1, seed=SEED, flags=fp.FP_FLAG_KEEP_HIDDEN)
             try:
                 fp.fp_prefill(h, toks, want_next=False)
-                got = fp.fp_get_tensor(h, fp.FP_G_HIDDEN, 0, 0, np.uint16, count=PREFIX * a.hidden)
-                got = quant.bf16_to_f32(got).reshape(PREFIX, a.hidden)
-                e = rel_err(got, ref)
-                assert e <= tau, (wq, kvq, B, ctx, e)
+                for b in sorted({0, B - 1}):
+                    got = fp.fp_get_tensor(h, fp.FP_G_HIDDEN, 0, 0, np.uint16, count=PREFIX * a.hidden,
+                                           offset=b * ctx * a.hidden)
+                    got = quant.bf16_to_f32(got).reshape(PREFIX, a.hidden)
+                    e = rel_err(got, ref)
+                    assert e <= tau, (wq, kvq, B, ctx, b, e)
                 r = fp.fp_profile(h, ctx, PROFILE_DECODE, warmup=0, iters=1, prompt=toks)
                 assert r.ttft_ms > 0 and r.tpot_ms > 0, (wq, kvq, B, ctx)
                 assert r.peak_hbm_bytes >= r.weight_bytes + r.kv_bytes, (wq, kvq, B, ctx)
