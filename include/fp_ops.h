@@ -126,6 +126,13 @@ int fp_op_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, 
                            size_t workspace_bytes, int32_t* err, void* stream);
 size_t fp_op_attention_decode_workspace_bytes(int B, int n_heads, int head_dim, int max_len);
 
+/* Context splits fp_op_attention_decode uses for B sequences, n_kv_heads KV
+ * heads and max_len cached positions (0 for a non-positive argument).  With
+ * 1 split the kernel normalises in place and never touches the workspace;
+ * with more, the partials go to the workspace and a second kernel merges
+ * them. */
+int fp_op_attention_decode_splits(int B, int n_kv_heads, int max_len);
+
 /* Decode attention without a caller workspace, for callers that cannot
  * allocate device memory (a host whose device memory is all reserved by
  * another framework's pool, a plugin that must not call the allocator, a
@@ -141,8 +148,11 @@ size_t fp_op_attention_decode_workspace_bytes(int B, int n_heads, int head_dim, 
  *     head_dim, max_len) exceeds FP_NOALLOC_SCRATCH_BYTES returns
  *     FP_ERR_UNSUPPORTED before anything is launched.
  *   - The first call on a device looks up the array's device address on that
- *     device (cudaGetSymbolAddress, with the device current) and caches it;
- *     make that first call before any stream capture.
+ *     device (cudaGetSymbolAddress, with the device current) and caches it
+ *     with the id of the device's current context; make that first call
+ *     before any stream capture.  After a device reset the context differs,
+ *     and the next call looks the address up again (make it, too, outside a
+ *     capture).
  *   - All calls share the one array, which keeps the last call's contents;
  *     each call writes every partial it reads back, so nothing needs
  *     clearing.  Calls that overlap on the GPU (other streams, other host

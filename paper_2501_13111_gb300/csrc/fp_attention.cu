@@ -104,6 +104,10 @@ int attention_decode_launches(int B, int n_kv_heads, int max_len) {
   return decode_geom(B, n_kv_heads, max_len).splits == 1 ? 1 : 2;
 }
 
+int attention_decode_splits(int B, int n_kv_heads, int max_len) {
+  return decode_geom(B, n_kv_heads, max_len).splits;
+}
+
 size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len) {
   const int tiles = std::max(1, (max_len + kDecTT - 1) / kDecTT);
   const size_t rows = (size_t)B * n_heads * dec_max_splits(B, tiles);

@@ -13,7 +13,13 @@
 // library's module is loaded holds FP_NOALLOC_SCRATCH_BYTES for it until the
 // process exits.  Host code cannot use the array's name as a device address
 // (on the host it names a host-side stand-in), so the device address is looked
-// up once per device with cudaGetSymbolAddress and cached.
+// up with cudaGetSymbolAddress, with the device current, and cached per device
+// together with the id of the context it was looked up in.  A device reset
+// (cudaDeviceReset) ends that context; the next call then runs in a new
+// context, whose id differs, and looks the address up again instead of using
+// one that belonged to the old context.
+#include <cuda.h>
+
 #include <mutex>
 
 #include "common.cuh"
@@ -27,22 +33,57 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-void* g_scratch_addr[kMaxDevices] = {};
+struct ScratchAddr {
+  void* ptr = nullptr;
+  unsigned long long ctx_id = 0;
+};
+ScratchAddr g_scratch_addr[kMaxDevices];
 
-// Device address of g_decode_scratch on the current device; looked up on the
-// first call for that device (with the device current) and cached.
+// Id of the calling thread's current context (unique over the process's
+// lifetime; cuCtxGetId), reached through the runtime's driver entry points so
+// that the library needs no link-time dependency on libcuda.  0 if unknown.
+unsigned long long current_context_id() {
+  typedef CUresult (*GetCurrentFn)(CUcontext*);
+  typedef CUresult (*GetIdFn)(CUcontext, unsigned long long*);
+  static GetCurrentFn get_current = nullptr;
+  static GetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPoint("cuCtxGetCurrent", &p, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = (GetCurrentFn)p;
+    p = nullptr;
+    if (cudaGetDriverEntryPoint("cuCtxGetId", &p, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = (GetIdFn)p;
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+// Device address of g_decode_scratch on the current device.  The first call
+// on a device (and the first after its context was replaced) looks it up and
+// caches it; a context whose id cannot be read is looked up on every call.
 int scratch_on_current_device(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return FP_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return FP_ERR_UNSUPPORTED;
+  const unsigned long long id = current_context_id();  // 0 before the runtime has made a context current
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_addr[dev]) {
+  ScratchAddr& a = g_scratch_addr[dev];
+  if (!a.ptr || id == 0 || a.ctx_id != id) {
     void* p = nullptr;
-    cudaError_t e = cudaGetSymbolAddress(&p, g_decode_scratch);
+    cudaError_t e = cudaGetSymbolAddress(&p, g_decode_scratch);  // with the device's primary context current
     if (e != cudaSuccess || !p) return FP_ERR_CUDA;
-    g_scratch_addr[dev] = p;
+    a.ptr = p;
+    a.ctx_id = id ? id : current_context_id();
   }
-  *out = g_scratch_addr[dev];
+  *out = a.ptr;
   return FP_OK;
 }
 
@@ -67,7 +108,8 @@ extern "C" int fp_op_attention_decode_noalloc(const uint16_t* q, int q_stride, i
   st = scratch_on_current_device(&scratch);
   if (st) return st;
   // Every partial the combine kernel reads is written by the same call, so the
-  // scratch needs no clearing between calls.
+  // scratch needs no clearing between calls.  Calls that overlap on the GPU
+  // share the array and race on it.
   cudaError_t e = fpk::launch_attention_decode(q, q_stride, B, n_heads, *kv, len, 0, max_len, out, scratch, err,
                                                (cudaStream_t)stream);
   return e == cudaSuccess ? FP_OK : FP_ERR_CUDA;

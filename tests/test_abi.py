@@ -189,3 +189,22 @@ def test_forward_kernels_wait_for_their_predecessor():
             if "pdl_wait()" not in src[body_start:i]:
                 missing.append(f"{name}:{kname}")
     assert not missing, missing
+
+
+def test_binding_constants_match_the_headers(fp):
+    """Constants the binding restates (the no-allocation scratch limit, the
+    layer cap) equal the header macros they copy."""
+    src = open(os.path.join(ROOT, "include", "fp_ops.h")).read() + open(os.path.join(ROOT, "include", "fp.h")).read()
+    m = re.search(r"#define\s+FP_NOALLOC_SCRATCH_BYTES\s+\((\d+)u\s*<<\s*(\d+)\)", src)
+    assert m, "FP_NOALLOC_SCRATCH_BYTES not found"
+    assert fp.FP_NOALLOC_SCRATCH_BYTES == int(m.group(1)) << int(m.group(2))
+    m = re.search(r"#define\s+FP_MAX_LAYERS\s+(\d+)", src)
+    assert fp.FP_MAX_LAYERS == int(m.group(1))
+
+
+def test_decode_splits_query_answers_on_host(fp):
+    """The split count is host arithmetic (no GPU call): one split for a short
+    context, several for the 70B-shaped decode attention."""
+    assert fp.fp_op_attention_decode_splits(0, 8, 100) == 0
+    assert fp.fp_op_attention_decode_splits(1, 1, 10) == 1
+    assert fp.fp_op_attention_decode_splits(2, 8, 2155) > 1
