@@ -2,16 +2,21 @@
 
 A step is one request batch through the whole hot path: prefill of the
 batch's prompts, then greedy decode steps (the decode step is a replayed CUDA
-graph).  The default workload is the Llama-2-7B-shaped fingerprint:
-2 decoder blocks (d 4096, 32 heads x 128, FFN 11008, vocab 32000), int8
-per-channel weight-only quantisation, bf16 KV cache, batch 8, 512-token
-prompts, 100 generated tokens.  Weights are synthetic (SplitMix64 /
-Irwin-Hall N(0, 0.02), drawn on the device), prompts are seeded uniform ids.
+graph).  The default workload is the largest configuration, the
+Llama-2-70B-shaped fingerprint: 2 decoder blocks (d 8192, 64 query / 8 KV
+heads x 128, FFN 28672, vocab 32000), int4 group-128 weight-only
+quantisation, int8 KV cache (per-token, per-head scales, 16-token pages),
+batch 32, 2048-token prompts, 100 generated tokens.  Weights are synthetic
+(SplitMix64 / Irwin-Hall N(0, 0.02), drawn on the device), prompts are
+seeded uniform ids.  --config picks the tiny, 7B- or 13B-shaped workload.
 
 value      decode tokens/s over all ranks = ranks * batch * decode steps / max-over-ranks
            device time of the decode phases (CUDA events on the library's stream)
-e2e        the same metric through the C ABI with host buffers: prompt H2D from
-           pinned memory each step and the token D2H after every decode step
+e2e        decode tokens/s of whole requests through the C ABI with host buffers:
+           each step uploads the prompt from pinned memory, prefills, reads the
+           first token back, and runs the decode steps with every step's input
+           tokens uploaded and its output tokens read back -- the prefill (TTFT)
+           is inside the timed region, as in the request latency of Eq. 1
 roofline   the dominant decode kernel: algorithmic bytes per launch / mean launch
            duration (CUDA events between kernels, instrumented decode steps)
 cpu_baseline  the oracle (numpy, fp64) on the host cores, a bounded sample
@@ -80,17 +85,18 @@ def kernel_bytes(a, wq, kvq, B, ctx):
 
 # ---------------------------------------------------------------- ncu traffic
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
-# 7B-shaped decode kernels from the ncu captures summarised in profiles/
-# (microbench cases 7b-*), with the sha256 prefix of the kernel's source at
-# capture time: a changed source makes the figure stale and it is reported as
-# null.  Attention traffic is per cached token row (captured at B 8, context
-# 612) and scales with B x context.
+# decode kernels from the ncu captures summarised in profiles/ (microbench
+# cases of the workload's shapes), keyed by (workload, kernel class), with the
+# sha256 prefix of the kernel's source at capture time: a changed source makes
+# the figure stale and it is reported as null.  Attention traffic is per
+# cached token row (units = B x context of the capture) and scales with the
+# bench's B x context.
 NCU_TRAFFIC = {
-    "attn": {"bytes": 81739520, "units": 8 * 612, "src": "fp_attention.cu", "sha": "de945a405c820013"},
-    "lm_head": {"bytes": 270745088, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-    "lin_gu": {"bytes": 94480640, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-    "lin_qkv": {"bytes": 50461184, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-    "lin_o": {"bytes": 16944384, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
+    ("l7b", "attn"): {"bytes": 81739520, "units": 8 * 612, "src": "fp_attention.cu", "sha": "de945a405c820013"},
+    ("l7b", "lm_head"): {"bytes": 270745088, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
+    ("l7b", "lin_gu"): {"bytes": 94480640, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
+    ("l7b", "lin_qkv"): {"bytes": 50461184, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
+    ("l7b", "lin_o"): {"bytes": 16944384, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
 }
 
 
@@ -98,8 +104,8 @@ def ncu_traffic(cls, cfg_name, B, ctx):
     """Per-launch DRAM bytes of kernel class `cls` from the recorded capture, or None."""
     import hashlib
 
-    t = NCU_TRAFFIC.get(cls)
-    if t is None or cfg_name != "l7b":
+    t = NCU_TRAFFIC.get((cfg_name, cls))
+    if t is None:
         return None
     src = os.path.join(ROOT, "paper_2501_13111_gb300", "csrc", t["src"])
     try:
@@ -204,12 +210,21 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- oracle timing
-def oracle_sample(cfg, batch, steps, decode_tokens, warmup=0):
-    """Time the oracle (numpy fp64, test infrastructure) on the same workload:
-    the full config shape at the same batch and prompt; the prompt's prefill
-    is set-up, each step is ``decode_tokens`` greedy decode steps, the first
-    ``warmup`` steps untimed.  Returns (tokens/s, seconds per timed step,
-    description)."""
+# The oracle's bounded sample of each workload: (batch, prompt) of the timed
+# decode.  The full shapes and the full batch are kept; where the workload's
+# prompt would make the untimed prefill set-up take minutes on the host
+# (the 70B-shaped prompt is 229 TFLOP at batch 32), a short prompt stands in.
+ORACLE_SAMPLE = {"tiny": (1, 32), "l7b": (8, 512), "l13b": (16, 64), "l70b": (32, 16)}
+
+
+def oracle_sample(cfg, batch, prompt, steps, decode_tokens, warmup=0):
+    """Time the oracle (numpy fp64, test infrastructure) on the workload's
+    shapes: the full config at ``batch`` sequences with ``prompt``-token
+    prompts; the prompt's prefill is set-up, each step is ``decode_tokens``
+    greedy decode steps, the first ``warmup`` steps untimed.  Returns
+    (tokens/s, seconds per timed step, description)."""
+    from concurrent.futures import ThreadPoolExecutor
+
     import synth
     from oracle import model as M
 
@@ -217,9 +232,10 @@ def oracle_sample(cfg, batch, steps, decode_tokens, warmup=0):
     arch = M.Arch(*t)
     get = lambda l, k, shape: (synth.f32_to_bf16_bits(np.ones(shape, np.float32)) if len(shape) == 1
                                else synth.weight_bf16(0, l, k, shape))
-    w, _ = M.build_weights(arch, wq, get)
-    ref = M.Fingerprint(arch, w, kvq, batch, S + (warmup + steps) * decode_tokens + 1)
-    toks = synth.tokens(0, batch * S, arch.vocab).reshape(batch, S)
+    with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as pool:  # set-up: quantise in parallel
+        w, _ = M.build_weights(arch, wq, get, map_fn=pool.map)
+    ref = M.Fingerprint(arch, w, kvq, batch, prompt + (warmup + steps) * decode_tokens + 1)
+    toks = synth.tokens(0, batch * prompt, arch.vocab).reshape(batch, prompt)
     out = ref.prefill(toks)
     tok = out["tokens"]
     times = []
@@ -230,8 +246,9 @@ def oracle_sample(cfg, batch, steps, decode_tokens, warmup=0):
         times.append(time.perf_counter() - t0)
     times = times[warmup:]
     tps = batch * decode_tokens * steps / sum(times)
-    desc = (f"oracle decode, batch {batch}, prompt {S} (prefill untimed), {decode_tokens} tokens x {steps} "
-            f"timed steps" + (f" after {warmup} untimed" if warmup else "") + ", fp64 numpy")
+    desc = (f"oracle decode of the full {arch.n_layers}-block shape, batch {batch} of {B}, prompt {prompt} of {S} "
+            f"(prefill untimed), {decode_tokens} tokens x {steps} timed steps"
+            + (f" after {warmup} untimed" if warmup else "") + ", fp64 numpy")
     return tps, times, desc
 
 
@@ -252,7 +269,8 @@ def run_reference(args, cfg):
     if int(os.environ.get("RANK", "0")) != 0:
         return 0
     t, wq, kvq, B, S, N = cfg
-    tps, times, desc = oracle_sample(cfg, B, args.steps, 2, warmup=args.warmup)
+    ob, op = ORACLE_SAMPLE[args.config]
+    tps, times, desc = oracle_sample(cfg, ob, op, args.steps, 2, warmup=args.warmup)
     line = {
         "metric": METRIC, "value": tps, "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
@@ -381,7 +399,7 @@ def main():
     ap.add_argument("--steps", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", default="l7b", choices=list(CONFIGS))
+    ap.add_argument("--config", default="l70b", choices=list(CONFIGS))
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing (profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass (profiling runs)")
     ap.add_argument("--sweep", action="store_true", help="profile the 96-point configuration sweep instead")
@@ -459,9 +477,10 @@ def main():
         block_gbs = [bb / (bm * 1e-3) / 1e9 for bb, bm in zip(prof["block_bytes"], prof["block_ms"])]
         launches = args.steps * (prof["prefill_launches"] + N * prof["decode_launches"])
 
-        # end to end through the C ABI with host buffers: every decode step
-        # takes its input tokens from pinned host memory and returns the
-        # generated ones there (the prompt's prefill is set-up, as above)
+        # end to end through the C ABI with host buffers: whole requests, the
+        # prompt uploaded from pinned host memory and prefilled, the first
+        # token read back, then every decode step's input tokens uploaded and
+        # its output tokens read back (Eq. 1's request latency, TTFT included)
         e2e = None
         if not args.no_e2e:
             pin_prompt = torch.empty((B, S), dtype=torch.int32, pin_memory=True)
@@ -473,8 +492,8 @@ def main():
             pin_out = torch.empty(B, dtype=torch.int32, pin_memory=True).numpy()
 
             def host_request():
-                fp.fp_prefill(h, host_prompt, out=pin_out)
                 t0 = time.perf_counter()
+                fp.fp_prefill(h, host_prompt, out=pin_out)
                 for _ in range(N):
                     pin_in[:] = pin_out
                     fp.fp_decode_step(h, pin_in, out=pin_out)
@@ -482,15 +501,17 @@ def main():
 
             host_request()
             barrier()
-            t_dec = sum(host_request() for _ in range(args.steps))
+            t_req = sum(host_request() for _ in range(args.steps))
             barrier()
-            t_dec = max_over_ranks(t_dec)
-            e2e = {"value": replica_tokens_per_s(world, B, N * args.steps, 1e3 * t_dec), "unit": "tokens/s",
-                   "h2d_bytes_per_step": B * 4 * N, "d2h_bytes_per_step": B * 4 * N}
+            t_req = max_over_ranks(t_req)
+            e2e = {"value": replica_tokens_per_s(world, B, N * args.steps, 1e3 * t_req), "unit": "tokens/s",
+                   "h2d_bytes_per_step": B * S * 4 + B * 4 * N, "d2h_bytes_per_step": B * 4 * (N + 1),
+                   "request_ms": 1e3 * t_req / args.steps, "covers": "prompt upload + prefill + decode steps"}
 
         cpu = None
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
-            tps, times, desc = oracle_sample(cfg, B, 2, 2)
+            ob, op = ORACLE_SAMPLE[args.config]
+            tps, times, desc = oracle_sample(cfg, ob, op, 3, 2)
             cpu = {"value": tps, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle", "sample": desc}
 
         if rank == 0:

@@ -4,11 +4,13 @@
 //
 // Two kernels, chosen by the number of rows M of x:
 //  * gemv_mma_kernel (M <= 64, decode): HBM-bound.  Each warp streams 16-row
-//    tiles of codes with 16-byte non-allocating loads, turns them into bf16
-//    MMA operands in registers (raw int8 codes, 128 + int4 codes), and runs
-//    mma.sync m16n8k16 against x staged once per CTA in shared memory.
-//    Scales are applied in fp32 (int8: per row in the epilogue; int4: per
-//    128-group, s * (acc - (128 + z) * sum x)), so the weights enter exactly.
+//    tiles of codes through a per-thread cp.async ring, turns them into MMA
+//    operands in registers, and runs mma.sync m16n8k16 against x staged
+//    once per window in shared memory.  bf16 weights enter as they are; int8
+//    and int4 codes become fp16(1152 + q) and fp16(1024 + q) by the exponent
+//    trick (exact), with x staged as fp16.  Offsets and scales are removed in
+//    fp32 (int8: acc - 1152 sum x, times the row scale in the epilogue; int4:
+//    per 128-group, s (acc - (1024 + z) sum x)), so the weights enter exactly.
 //    The (row block, K step) work is cut into equal contiguous ranges, one
 //    per resident CTA; a row block shared by several CTAs is finished by the
 //    last of them from fp32 partials (no spinning).
