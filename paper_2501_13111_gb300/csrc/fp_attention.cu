@@ -478,6 +478,318 @@ __global__ void attn_combine_kernel(int H, const int32_t* __restrict__ len, int 
   out[(long long)bh * HD + e] = f2bf(o / L);
 }
 
+// =====================================================================
+// Decode attention over an int8 cache, head_dim 128, 16-token pages: each
+// warp streams whole pages of its KV head on its own.
+//
+// CTA = one (sequence, KV head, context split), 4 warps; warp w takes pages
+// w, w + 4, ... of the split.  A page of one KV head is 2 KB of K codes, 2 KB
+// of V codes and 2 x 64 B of scales, contiguous in the pool; each warp copies
+// its pages into a private 3-page cp.async ring (16-byte chunks, row r's
+// chunk c stored at c ^ (r & 7) so the reads below are conflict-free) and
+// waits only for its own copies: no CTA barrier inside the loop.
+//
+// Per page, two MMA passes (mma.sync m16n8k16, fp16 in, fp32 accumulate):
+//   S^T = K Q^T: A = the page's 16 keys x 16 dims, B = Q^T (16 dims x the
+//     G <= 8 query heads of the KV head): the heads fill the N = 8 of the
+//     instruction.  The dims are permuted so that thread (g, t) reads 32
+//     consecutive code bytes of keys g and g + 8 -- k-step ks, slots
+//     (2t, 2t+1, 2t+8, 2t+9) <-> dims 32t + 4ks + (0, 1, 2, 3) -- and Q is
+//     loaded with the same permutation once per CTA.
+//   O^T += V^T P'^T: A = 16 dims x the page's 16 tokens (thread (g, t) owns
+//     dims 16g .. 16g + 15, so it reads one 16-byte chunk of each of its four
+//     tokens; m-tile mt holds dims 16g + 2mt and 16g + 2mt + 1), B = P' (the
+//     probabilities times each token's V scale) of 16 tokens x 8 heads, moved
+//     from the S^T accumulator layout by four shuffles.
+// Codes enter as fp16(1152 + q) (a byte permute with 0x64 high bytes after
+// q ^ 0x80, exact); the offset is removed in fp32: scores subtract
+// 1152 sum_d Q[h][d], outputs 1152 sum_t P'[t][h].  Online softmax in the
+// log2 domain per head, the K scales multiplying the score columns.  The
+// warps are merged in shared memory at the end; the result is normalised in
+// place (one split) or written as (o, m, l) for attn_combine_kernel.
+// =====================================================================
+constexpr int kD8Warps = 4, kD8Stages = 3;
+constexpr int kD8PageBytes = 2 * 16 * 128 + 2 * 16 * 4;  // K and V codes, then K and V scales
+
+FP_DEV uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t r;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+  return r;
+}
+FP_DEV uint4 lds128(const uint8_t* p) { return *reinterpret_cast<const uint4*>(p); }
+FP_DEV uint32_t word4(const uint4& v, int i) { return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w; }
+
+constexpr size_t d8_smem_bytes(int chunk) {
+  return (size_t)kD8Warps * kD8Stages * kD8PageBytes + ((size_t)chunk / 16 + 2) * sizeof(int);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kD8Warps * 32) attn_decode_i8_kernel(
+    const uint16_t* __restrict__ q, int q_stride, int H, fp_kv_view kv, const int32_t* __restrict__ len,
+    int len_add, int max_len, int chunk, int splits, float* __restrict__ ws, uint16_t* __restrict__ out,
+    int32_t* err) {
+  constexpr int HD = 128;
+  extern __shared__ __align__(16) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+  pdl_trigger();
+  pdl_wait();
+  const int Hkv = kv.n_kv_heads;
+  const int b = blockIdx.x / Hkv, kvh = blockIdx.x % Hkv;
+  const int split = blockIdx.y;
+  int T = len[b] + len_add;
+  if (T > max_len) {  // never past the positions the grid and the page table cover
+    if (err && split == 0 && threadIdx.x == 0) atomicExch(err, 1);
+    T = max_len;
+  }
+  const int t0 = split * chunk;
+  if (t0 >= T) {
+    if (splits == 1)  // empty context: zero output
+      for (int i = threadIdx.x; i < G * HD; i += blockDim.x) out[((long long)b * H + kvh * G) * HD + i] = 0;
+    return;
+  }
+  const int t1 = min(T, t0 + chunk);
+  const int np = (t1 - t0 + 15) / 16;  // pages of the split (t0 is a multiple of 64)
+  // ---- the split's page ids, staged once (past the table: -1)
+  int* spt = reinterpret_cast<int*>(smem + kD8Warps * kD8Stages * kD8PageBytes);
+  {
+    const int32_t* pt = kv.page_table + (long long)b * kv.pages_per_seq;
+    const int lp0 = t0 / 16;
+    for (int i = threadIdx.x; i < np; i += blockDim.x) spt[i] = lp0 + i < kv.pages_per_seq ? pt[lp0 + i] : -1;
+    __syncthreads();
+  }
+  uint8_t* ring = smem + warp * kD8Stages * kD8PageBytes;
+
+  // ---- copy page j of this warp (split page warp + 4 j) into ring slot j % 3
+  auto issue = [&](int j) {
+    const int pi = warp + kD8Warps * j;
+    uint8_t* dst = ring + (j % kD8Stages) * kD8PageBytes;
+    if (pi < np) {
+      const int page = spt[pi];
+      if (page >= 0 && page < kv.n_pages) {
+        const long long row0 = ((long long)page * Hkv + kvh) * 16;  // first token row of (page, head)
+        const uint8_t* kg = (const uint8_t*)kv.k_pool + row0 * HD;
+        const uint8_t* vg = (const uint8_t*)kv.v_pool + row0 * HD;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int c = lane + 32 * i, r = c >> 3, cc = c & 7;
+          const int off = r * HD + ((cc ^ (r & 7)) << 4);
+          dec_cp_async16(dst + off, kg + c * 16);
+          dec_cp_async16(dst + 2048 + off, vg + c * 16);
+        }
+        if (lane < 4) dec_cp_async16(dst + 4096 + lane * 16, (const uint8_t*)(kv.k_scale + row0) + lane * 16);
+        else if (lane < 8) dec_cp_async16(dst + 4160 + (lane - 4) * 16, (const uint8_t*)(kv.v_scale + row0) + (lane - 4) * 16);
+      } else {
+        // a bad page id reads as zero codes and zero scales
+        if (err && lane == 0) atomicExch(err, 1);
+        for (int i = lane; i < kD8PageBytes / 16; i += 32) *reinterpret_cast<uint4*>(dst + i * 16) = make_uint4(0, 0, 0, 0);
+      }
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  const int nj = np > warp ? (np - warp + kD8Warps - 1) / kD8Warps : 0;  // this warp's pages
+#pragma unroll
+  for (int j = 0; j < kD8Stages - 1; ++j) issue(j);
+
+  // ---- Q^T as the B operand (head g, dims 32t + 4ks + 0..3), fp16; and
+  // sum_d Q[h][d] of the fp16 values for the heads 2t, 2t + 1 of this thread
+  uint32_t qb[8][2];
+  float qsum = 0.f;
+  {
+    const uint16_t* qh = q + (long long)b * q_stride + (long long)(kvh * G + g) * HD + 32 * t;
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t lo = 0, hi = 0;
+      if (g < G) {  // q_stride may be odd: 16-bit loads
+        const uint16_t* qp = qh + 4 * ks;
+        const __half2 a = __floats2half2_rn(bf2f(qp[0]), bf2f(qp[1]));
+        const __half2 c = __floats2half2_rn(bf2f(qp[2]), bf2f(qp[3]));
+        const float2 fa = __half22float2(a), fc = __half22float2(c);
+        qsum += (fa.x + fa.y) + (fc.x + fc.y);
+        lo = *reinterpret_cast<const uint32_t*>(&a);
+        hi = *reinterpret_cast<const uint32_t*>(&c);
+      }
+      qb[ks][0] = lo;
+      qb[ks][1] = hi;
+    }
+    qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
+    qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
+  }
+  // lanes 4h .. 4h + 3 hold head h's sum; this thread's score columns are heads 2t, 2t + 1
+  const float qoff0 = 1152.f * __shfl_sync(0xffffffffu, qsum, 8 * t);
+  const float qoff1 = 1152.f * __shfl_sync(0xffffffffu, qsum, 8 * t + 4);
+  const float scale = kLog2e * rsqrtf((float)HD);
+
+  float o[8][4];  // O^T: m-tile mt rows (dims 16g + 2mt, 16g + 2mt + 1) x heads (2t, 2t + 1)
+#pragma unroll
+  for (int i = 0; i < 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m[2] = {-INFINITY, -INFINITY}, l[2] = {0.f, 0.f}, sp[2] = {0.f, 0.f};  // heads 2t, 2t + 1
+  const uint32_t sw = (uint32_t)(g & 7);
+
+  for (int j = 0; j < nj; ++j) {
+    asm volatile("cp.async.wait_group %0;" ::"n"(kD8Stages - 2) : "memory");
+    __syncwarp();  // every lane's copies of page j landed; the slot refilled below was read last round
+    issue(j + kD8Stages - 1);
+    const uint8_t* pg = ring + (j % kD8Stages) * kD8PageBytes;
+    const int tok0 = t0 + (warp + kD8Warps * j) * 16;
+
+    // ---- S^T = K Q^T over the page's 16 tokens
+    float s[4] = {0.f, 0.f, 0.f, 0.f};  // (token g | g + 8) x (head 2t | 2t + 1)
+    {
+      const uint4 ka0 = lds128(pg + g * HD + (((2 * t) ^ sw) << 4));
+      const uint4 ka1 = lds128(pg + g * HD + (((2 * t + 1) ^ sw) << 4));
+      const uint4 kb0 = lds128(pg + (g + 8) * HD + (((2 * t) ^ sw) << 4));
+      const uint4 kb1 = lds128(pg + (g + 8) * HD + (((2 * t + 1) ^ sw) << 4));
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        const uint32_t wa = word4(ks < 4 ? ka0 : ka1, ks & 3) ^ 0x80808080u;
+        const uint32_t wb = word4(ks < 4 ? kb0 : kb1, ks & 3) ^ 0x80808080u;
+        const uint32_t a[4] = {prmt(wa, 0x64646464u, 0x5140), prmt(wb, 0x64646464u, 0x5140),
+                               prmt(wa, 0x64646464u, 0x5342), prmt(wb, 0x64646464u, 0x5342)};
+        dec_mma<true>(s, a, qb[ks][0], qb[ks][1]);
+      }
+    }
+    // ---- scores (log2 domain): s_k[token] (S^T - 1152 sum Q) / sqrt(hd); tokens past t1 masked
+    const float* ksc = reinterpret_cast<const float*>(pg + 4096);
+    const float* vsc = reinterpret_cast<const float*>(pg + 4160);
+    const bool ok_lo = tok0 + g < t1, ok_hi = tok0 + g + 8 < t1;
+    const float sk_lo = ksc[g] * scale, sk_hi = ksc[g + 8] * scale;
+    float sc[4];
+    sc[0] = ok_lo ? (s[0] - qoff0) * sk_lo : -INFINITY;
+    sc[1] = ok_lo ? (s[1] - qoff1) * sk_lo : -INFINITY;
+    sc[2] = ok_hi ? (s[2] - qoff0) * sk_hi : -INFINITY;
+    sc[3] = ok_hi ? (s[3] - qoff1) * sk_hi : -INFINITY;
+    uint32_t pk[2];  // fp16 pairs (P'[token g][head 2t + e], P'[token g + 8][head 2t + e])
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      float mx = fmaxf(sc[e], sc[2 + e]);
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+      const float mnew = fmaxf(m[e], mx);
+      const float ref = mnew == -INFINITY ? 0.f : mnew;
+      const float corr = exp2f(m[e] - ref);
+      const float p_lo = exp2f(sc[e] - ref), p_hi = exp2f(sc[2 + e] - ref);
+      l[e] = l[e] * corr + p_lo + p_hi;
+      m[e] = mnew;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        o[mt][e] *= corr;
+        o[mt][2 + e] *= corr;
+      }
+      // P' = P times the token's V scale (zero for masked tokens), rounded to fp16;
+      // the V offset uses the sum of the rounded values
+      const __half2 pp = __floats2half2_rn(ok_lo ? p_lo * vsc[g] : 0.f, ok_hi ? p_hi * vsc[g + 8] : 0.f);
+      const float2 pr = __half22float2(pp);
+      sp[e] = sp[e] * corr + pr.x + pr.y;
+      pk[e] = *reinterpret_cast<const uint32_t*>(&pp);
+    }
+    // ---- P'^T as the B operand: thread (g, t) needs head g at tokens 2t, 2t + 1
+    // (from lane 8t + g/2) and 2t + 8, 2t + 9 (lane 8t + 4 + g/2), parity g & 1
+    uint32_t pb0, pb1;
+    {
+      const int l0 = 8 * t + (g >> 1), l1 = l0 + 4;
+      const uint32_t a0 = __shfl_sync(0xffffffffu, pk[0], l0), a1 = __shfl_sync(0xffffffffu, pk[1], l0);
+      const uint32_t c0 = __shfl_sync(0xffffffffu, pk[0], l1), c1 = __shfl_sync(0xffffffffu, pk[1], l1);
+      const uint32_t v0 = (g & 1) ? a1 : a0, v1 = (g & 1) ? c1 : c0;  // (tok 2t | 2t+8), (tok 2t+1 | 2t+9)
+      pb0 = prmt(v0, v1, 0x5410);  // tokens 2t, 2t + 1
+      pb1 = prmt(v0, v1, 0x7632);  // tokens 2t + 8, 2t + 9
+    }
+    // ---- O^T += V^T P'^T: thread (g, t) reads dims 16g .. 16g + 15 of tokens 2t, 2t + 1, 2t + 8, 2t + 9
+    {
+      const uint4 va = lds128(pg + 2048 + (2 * t) * HD + ((g ^ ((2 * t) & 7)) << 4));
+      const uint4 vb = lds128(pg + 2048 + (2 * t + 1) * HD + ((g ^ ((2 * t + 1) & 7)) << 4));
+      const uint4 vc = lds128(pg + 2048 + (2 * t + 8) * HD + ((g ^ ((2 * t + 8) & 7)) << 4));
+      const uint4 vd = lds128(pg + 2048 + (2 * t + 9) * HD + ((g ^ ((2 * t + 9) & 7)) << 4));
+#pragma unroll
+      for (int wi = 0; wi < 4; ++wi) {
+        const uint32_t A = word4(va, wi) ^ 0x80808080u, Bw = word4(vb, wi) ^ 0x80808080u;
+        const uint32_t C = word4(vc, wi) ^ 0x80808080u, D = word4(vd, wi) ^ 0x80808080u;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {  // m-tile 2 wi + h: bytes 2h, 2h + 1 of the words
+          const uint32_t xab = prmt(A, Bw, h ? 0x7362 : 0x5140), xcd = prmt(C, D, h ? 0x7362 : 0x5140);
+          const uint32_t a[4] = {prmt(xab, 0x64646464u, 0x5140), prmt(xab, 0x64646464u, 0x5342),
+                                 prmt(xcd, 0x64646464u, 0x5140), prmt(xcd, 0x64646464u, 0x5342)};
+          dec_mma<true>(o[2 * wi + h], a, pb0, pb1);
+        }
+      }
+    }
+  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+#pragma unroll
+    for (int x = 4; x <= 16; x <<= 1) {
+      l[e] += __shfl_xor_sync(0xffffffffu, l[e], x);
+      sp[e] += __shfl_xor_sync(0xffffffffu, sp[e], x);
+    }
+  }
+  __syncthreads();  // the rings are reused for the merge below
+
+  // ---- merge the 4 warps: per head, o = sum_w o_w 2^(m_w - M), l = sum_w l_w 2^(m_w - M)
+  float* red = reinterpret_cast<float*>(smem);  // [4][8][HD + 2]
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const int hh = 2 * t + e;
+    if (hh < G) {
+      float* r = red + (warp * 8 + hh) * (HD + 2);
+      const float off = 1152.f * sp[e];
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        r[16 * g + 2 * mt] = o[mt][e] - off;
+        r[16 * g + 2 * mt + 1] = o[mt][2 + e] - off;
+      }
+      if (g == 0) {
+        r[HD] = m[e];
+        r[HD + 1] = l[e];
+      }
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < G * HD; i += blockDim.x) {
+    const int hh = i / HD, e = i % HD;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kD8Warps; ++w) M = fmaxf(M, red[(w * 8 + hh) * (HD + 2) + HD]);
+    float ov = 0.f, L = 0.f;
+#pragma unroll
+    for (int w = 0; w < kD8Warps; ++w) {
+      const float* r = red + (w * 8 + hh) * (HD + 2);
+      const float f = r[HD] == -INFINITY ? 0.f : exp2f(r[HD] - M);
+      ov += r[e] * f;
+      L += r[HD + 1] * f;
+    }
+    if (splits == 1) {  // the whole context: normalise here, no combine pass
+      out[((long long)b * H + kvh * G + hh) * HD + e] = f2bf(ov / L);
+      continue;
+    }
+    const long long row = ((long long)b * H + kvh * G + hh) * splits + split;
+    float* w = ws + row * (HD + 2);
+    w[e] = ov;
+    if (e == 0) {
+      w[HD] = M;
+      w[HD + 1] = L;
+    }
+  }
+}
+
+template <int G>
+static cudaError_t launch_decode_i8(const uint16_t* q, int q_stride, int B, int H, const fp_kv_view& kv,
+                                    const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
+                                    uint16_t* out, int32_t* err, cudaStream_t s, cudaError_t* second) {
+  const size_t smem = d8_smem_bytes(g.chunk);
+  auto kern = attn_decode_i8_kernel<G>;
+  static std::atomic<unsigned long long> attr{0};
+  FP_CUDA_TRY(smem_limit_once(kern, (int)d8_smem_bytes(kDecMaxChunkTiles * kDecTT), &attr));
+  dim3 grid(B * kv.n_kv_heads, g.splits);
+  cudaError_t e = launch(kern, grid, dim3(kD8Warps * 32), smem, s, q, q_stride, H, kv, len, len_add, max_len,
+                         g.chunk, g.splits, ws, out, err);
+  if (e != cudaSuccess || g.splits == 1) return e;
+  e = launch(attn_combine_kernel<128>, dim3(B * H), dim3(128), 0, s, H, len, len_add, max_len, g.chunk, g.splits,
+             (const float*)ws, out);
+  if (second) *second = e;
+  return e;
+}
+
 template <int HD, int KVQ, int G, int NB>
 static cudaError_t launch_decode_nb(const uint16_t* q, int q_stride, int B, int H, const fp_kv_view& kv,
                                     const int32_t* len, int len_add, int max_len, DecodeGeom g, float* ws,
@@ -523,6 +835,16 @@ cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int 
   DecodeGeom g = decode_geom(B, kv.n_kv_heads, max_len);
   const int G = n_heads / kv.n_kv_heads;
   float* w = (float*)ws;
+  const bool a16 = (((uintptr_t)kv.k_pool | (uintptr_t)kv.v_pool | (uintptr_t)kv.k_scale | (uintptr_t)kv.v_scale) & 15) == 0;
+  if (kv.kvquant == FP_KV_INT8 && kv.head_dim == 128 && kv.page_size == 16 && a16) {
+    switch (G) {
+      case 1: return launch_decode_i8<1>(q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second);
+      case 2: return launch_decode_i8<2>(q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second);
+      case 4: return launch_decode_i8<4>(q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second);
+      case 8: return launch_decode_i8<8>(q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   if (kv.head_dim == 64) {
     return kv.kvquant == FP_KV_BF16
                ? launch_decode_g<64, FP_KV_BF16>(G, q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second)
