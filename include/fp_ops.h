@@ -172,6 +172,17 @@ int fp_op_attention_decode_noalloc(const uint16_t* q, int q_stride, int B, int n
 int fp_op_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
                             const fp_kv_view* kv, uint16_t* out, int32_t* err, void* stream);
 
+/* Test hook for the failure path of the pipelined tensor-core kernels (the
+ * paper has no counterpart).  Every wait of those kernels is bounded; a role
+ * whose wait runs out stops, the CTA drains its copies and MMAs in flight,
+ * frees its tensor memory and records status 2 in the error word, which the
+ * runtime reports as FP_ERR_DEVICE_ASSERT.  This sets how many polling rounds
+ * the prefill GEMM's MMA thread waits for a stage of operands on the current
+ * device: rounds >= 0 (0 gives up at once) or < 0 to restore the default;
+ * all other waits keep the default.  Synchronous; not for use while kernels
+ * of the library are running. */
+int fp_debug_set_wait_limit(long long rounds);
+
 /* Greedy choice out[m] = argmax logits[m][:V] (fp32); ties to the lowest id. */
 int fp_op_argmax(const float* logits, int M, int V, int32_t* out, void* stream);
 

@@ -145,6 +145,7 @@ _PROTOS = {
     "fp_op_attention_decode_noalloc": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _P]),
     "fp_op_attention_prefill": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P]),
     "fp_op_argmax": (_I, [_P, _I, _I, _P, _P]),
+    "fp_debug_set_wait_limit": (_I, [_LL]),
     "fp_solve_eq1": (_I, [_I, C.c_double, _I, C.c_double, C.POINTER(fp_eq1_fit)]),
     "fp_solve_eq23": (_I, [_I, C.POINTER(fp_eq1_fit), _I, C.POINTER(fp_eq1_fit), C.POINTER(fp_l2_terms)]),
     "fp_predict_latency": (_I, [C.POINTER(fp_l2_terms), _I, _I, C.POINTER(C.c_double)]),
@@ -338,6 +339,11 @@ def fp_op_attention_prefill(q, q_stride, B, S, n_heads, kv: fp_kv_view, out, err
 
 def fp_op_argmax(logits, M, V, out, stream=None):
     return _check(_lib.fp_op_argmax(logits, M, V, out, stream))
+
+
+def fp_debug_set_wait_limit(rounds):
+    """Test hook: polling rounds of the prefill GEMM's stage wait (< 0: default)."""
+    return _check(_lib.fp_debug_set_wait_limit(rounds))
 
 
 # ------------------------------------------------------------------ torch plumbing

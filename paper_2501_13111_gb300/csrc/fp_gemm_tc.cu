@@ -29,6 +29,12 @@
 #include "kernels.cuh"
 #include "tc.cuh"
 
+// Rounds after which the MMA thread's wait for a stage gives up: kTcSpinLimit,
+// unless a test lowers it through fp_debug_set_wait_limit to run the failure
+// path (every other wait keeps kTcSpinLimit, so copies and MMAs in flight are
+// still drained before the CTA leaves).
+static __device__ long long g_stage_wait_limit = fpk::kTcSpinLimit;
+
 namespace fpk {
 
 constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64, kTcStages = 4;
@@ -130,6 +136,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // ---------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = tc_idesc(kTcBM, kTcBN);
+      const long long stage_limit = g_stage_wait_limit;
       int it = 0, lt = 0;
       for (int t = blockIdx.x; t < ntiles && !*abort_flag; t += gridDim.x, ++lt) {
         const int acc = lt & 1;
@@ -144,7 +151,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         bool ok = true;
         for (int kb = 0; kb < kblocks; ++kb, ++it) {
           const int s = it % kTcStages;
-          if (!mbar_wait(&full[s], (it / kTcStages) & 1) || *abort_flag) {
+          if (!mbar_wait_n(&full[s], (it / kTcStages) & 1, stage_limit) || *abort_flag) {
             ok = false;
             break;
           }
@@ -381,3 +388,8 @@ cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N,
 }
 
 }  // namespace fpk
+
+extern "C" int fp_debug_set_wait_limit(long long rounds) {
+  const long long v = rounds < 0 ? fpk::kTcSpinLimit : std::min(rounds, fpk::kTcSpinLimit);
+  return cudaMemcpyToSymbol(g_stage_wait_limit, &v, sizeof v) == cudaSuccess ? FP_OK : FP_ERR_CUDA;
+}

@@ -200,9 +200,11 @@ static cudaError_t launch_gemv(int epi, const uint16_t* x, int M, int N, int K, 
 // Operands: bf16 weights multiply bf16 x as they are.  int8 and int4 codes
 // become fp16 by the 0x6400 exponent trick -- fp16(1152 + q) for int8,
 // fp16(1024 + q) for int4, both exact -- and x is staged as fp16 (exact
-// for |x| in the fp16 normal range; |x| >= 65504 is not supported).  The
-// offsets are removed in fp32: int8 acc - 1152 * sum(x) over the CTA's K
-// range, int4 per 128-group s * (acc - (1024 + z) * sum(x)).
+// for |x| in the fp16 normal range; smaller values become fp16 subnormals,
+// and an |x| that rounds beyond 65504 becomes inf and sets the error word to
+// 3, which the runtime reports).  The offsets are removed in fp32: int8
+// acc - 1152 * sum(x) over the CTA's K range, int4 per 128-group
+// s * (acc - (1024 + z) * sum(x)).
 template <int WQ>
 struct MmaFmt;
 template <>
@@ -312,7 +314,8 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_mma_kernel(const uint16_
                                                        const uint16_t* __restrict__ scales,
                                                        const uint16_t* __restrict__ zeros, const uint16_t* R,
                                                        void* Y, long long total, int S, int W,
-                                                       float* __restrict__ ws, unsigned* __restrict__ counters) {
+                                                       float* __restrict__ ws, unsigned* __restrict__ counters,
+                                                       int32_t* err) {
   constexpr int KT = MmaFmt<WQ>::KT, SUP = 4 * KT, KS = KT / 4, CH = KT / 8;
   constexpr bool F16 = WQ != FP_W_BF16;
   constexpr bool G128 = WQ == FP_W_INT4_G128;
@@ -429,11 +432,14 @@ __global__ void __launch_bounds__(kGemvWarps * 32) gemv_mma_kernel(const uint16_
           if constexpr (F16) {
             const uint32_t w4[4] = {xo.x, xo.y, xo.z, xo.w};
             float sum = 0.f;
+            bool over = false;
 #pragma unroll
             for (int p = 0; p < 4; ++p) {
               const float2 f = x_pair<WQ>(w4[p]);
               sum += f.x + f.y;
+              over |= isinf(f.x) || isinf(f.y);
             }
+            if (over && err) atomicExch(err, 3);  // x outside the fp16 range: the output is invalid
             // the 4 lanes of one x row (same g) hold consecutive pieces of it
             sum += __shfl_xor_sync(0xffffffffu, sum, 1);
             sum += __shfl_xor_sync(0xffffffffu, sum, 2);
@@ -749,7 +755,7 @@ static GemvPlan plan_for(int wq, int epi, int M, int N, int K) {
 template <int WQ, int NT, int EPI>
 static cudaError_t launch_mma_t(const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
                                 const uint16_t* zeros, const uint16_t* R, void* y, void* ws, size_t ws_bytes,
-                                cudaStream_t s) {
+                                cudaStream_t s, int32_t* err) {
   const GemvPlan p = plan_t<WQ, NT, EPI>(M, N, K);
   if (p.ctas <= 0) return cudaErrorInvalidValue;
   // never launch with less workspace than this plan writes; partials are read as float4
@@ -757,30 +763,30 @@ static cudaError_t launch_mma_t(const uint16_t* x, int M, int N, int K, const vo
   unsigned* counters = (unsigned*)ws;
   float* part = (float*)((char*)ws + counter_bytes(p.blocks));
   return launch(gemv_mma_kernel<WQ, NT, EPI>, dim3(p.ctas), dim3(kGemvWarps * 32), p.smem, s, x, M, N, K, codes,
-                scales, zeros, R, y, p.total, p.S, p.W, part, counters);
+                scales, zeros, R, y, p.total, p.S, p.W, part, counters, err);
 }
 
 template <int WQ, int EPI>
 static cudaError_t launch_mma_e(const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
                                 const uint16_t* zeros, const uint16_t* R, void* y, void* ws, size_t ws_bytes,
-                                cudaStream_t s) {
+                                cudaStream_t s, int32_t* err) {
   switch (gemv_nt(M)) {
-    case 1: return launch_mma_t<WQ, 1, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    case 2: return launch_mma_t<WQ, 2, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    case 4: return launch_mma_t<WQ, 4, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    default: return launch_mma_t<WQ, 8, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case 1: return launch_mma_t<WQ, 1, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
+    case 2: return launch_mma_t<WQ, 2, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
+    case 4: return launch_mma_t<WQ, 4, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
+    default: return launch_mma_t<WQ, 8, EPI>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
   }
 }
 
 template <int WQ>
 static cudaError_t launch_mma(int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                               const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* y, void* ws,
-                              size_t ws_bytes, cudaStream_t s) {
+                              size_t ws_bytes, cudaStream_t s, int32_t* err) {
   switch (epi) {
-    case FP_EPI_STORE: return launch_mma_e<WQ, FP_EPI_STORE>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    case FP_EPI_RESID: return launch_mma_e<WQ, FP_EPI_RESID>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    case FP_EPI_SWIGLU: return launch_mma_e<WQ, FP_EPI_SWIGLU>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
-    default: return launch_mma_e<WQ, FP_EPI_F32>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s);
+    case FP_EPI_STORE: return launch_mma_e<WQ, FP_EPI_STORE>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
+    case FP_EPI_RESID: return launch_mma_e<WQ, FP_EPI_RESID>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
+    case FP_EPI_SWIGLU: return launch_mma_e<WQ, FP_EPI_SWIGLU>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
+    default: return launch_mma_e<WQ, FP_EPI_F32>(x, M, N, K, codes, scales, zeros, R, y, ws, ws_bytes, s, err);
   }
 }
 
@@ -828,9 +834,9 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
     return launch_q4tc(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, err, s);
   if (mma_ok(wquant, M, N, K)) {
     switch (wquant) {
-      case FP_W_BF16: return launch_mma<FP_W_BF16>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s);
-      case FP_W_INT8: return launch_mma<FP_W_INT8>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s);
-      default: return launch_mma<FP_W_INT4_G128>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s);
+      case FP_W_BF16: return launch_mma<FP_W_BF16>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s, err);
+      case FP_W_INT8: return launch_mma<FP_W_INT8>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s, err);
+      default: return launch_mma<FP_W_INT4_G128>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s, err);
     }
   }
   switch (wquant) {

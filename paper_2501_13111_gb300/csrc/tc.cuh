@@ -37,6 +37,23 @@ FP_DEV bool mbar_wait(uint64_t* bar, uint32_t parity) {
   return false;
 }
 
+// As mbar_wait, giving up after `limit` rounds (at most kTcSpinLimit); limit
+// 0 gives up at once.
+FP_DEV bool mbar_wait_n(uint64_t* bar, uint32_t parity, long long limit) {
+  const uint32_t a = smem_u32(bar);
+  for (long long it = 0; it < kTcSpinLimit; ++it) {
+    if (it >= limit) return false;
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(done)
+        : "r"(a), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+
 // As mbar_wait, but a thread that finds the phase still open sleeps a little
 // before it polls again, so many waiting warps leave the issue slots to the
 // warps that have work.

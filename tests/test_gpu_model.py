@@ -206,3 +206,58 @@ def test_profile_reports(fp):
         assert r.peak_hbm_bytes >= r.weight_bytes + r.kv_bytes
     finally:
         fp.fp_destroy(h)
+
+
+def test_fp16_overflow_in_decode_linear_is_reported(fp):
+    """The decode GEMV stages x as fp16 for int8 / int4 weights.  An
+    activation beyond the fp16 range (here a pre-attention norm gain of
+    about 1e5 makes |y| > 65504) must not pass silently: the step returns
+    FP_ERR_DEVICE_ASSERT and says why; a later step with sane gains is clean."""
+    arch = M.Arch(1, 512, 8, 8, 64, 1376, 32000)
+    h = fp.fp_create(arch_dict(arch), 1, 0, 2, 64, seed=9)
+    try:
+        toks = synth.tokens(9, 2 * 40, arch.vocab).reshape(2, 40)
+        fp.fp_prefill(h, toks)
+        big = synth.f32_to_bf16_bits(np.full(arch.hidden, 1e5, np.float32))
+        fp.fp_set_weight(h, 0, fp.FP_T_ATTN_NORM, big)
+        with pytest.raises(fp.FPError) as e:
+            fp.fp_decode_step(h, np.array([1, 2], np.int32))
+        assert e.value.code == fp.FP_ERR_DEVICE_ASSERT
+        assert "fp16" in str(e.value)
+        fp.fp_set_weight(h, 0, fp.FP_T_ATTN_NORM, synth.f32_to_bf16_bits(np.ones(arch.hidden, np.float32)))
+        fp.fp_prefill(h, toks)
+        fp.fp_decode_step(h, np.array([1, 2], np.int32))  # clean again: the error word was cleared
+    finally:
+        fp.fp_destroy(h)
+
+
+def test_expired_wait_in_the_tcgen05_gemm_is_reported(fp):
+    """The failure path of the pipelined tensor-core kernels, without a fault:
+    the test lowers the prefill GEMM's stage wait to zero rounds, so its MMA
+    thread gives up at the first stage; the CTA drains what it issued, frees
+    its tensor memory and records status 2.  The prefill then returns
+    FP_ERR_DEVICE_ASSERT, and with the default restored the same handle runs
+    clean and matches the oracle."""
+    arch = M.Arch(1, 512, 8, 8, 64, 1376, 32000)
+    B, S = 2, 40  # 80 prompt rows: the prefill linears run on the tcgen05 GEMM
+    get = weight_getter(13)
+    w, _ = M.build_weights(arch, 0, get)
+    h = fp.fp_create(arch_dict(arch), 0, 0, B, 64, flags=fp.FP_FLAG_NO_INIT)
+    try:
+        upload_weights(fp, h, arch, get)
+        toks = synth.tokens(13, B * S, arch.vocab).reshape(B, S)
+        fp.fp_debug_set_wait_limit(0)
+        try:
+            with pytest.raises(fp.FPError) as e:
+                fp.fp_prefill(h, toks)
+        finally:
+            fp.fp_debug_set_wait_limit(-1)
+        assert e.value.code == fp.FP_ERR_DEVICE_ASSERT
+        assert "bounded wait" in str(e.value)
+        nxt = fp.fp_prefill(h, toks)
+        out = M.Fingerprint(arch, w, 0, B, 64).prefill(toks)
+        lg = fp.fp_get_tensor(h, fp.FP_G_LOGITS, 0, 0, np.float32).reshape(B, -1)
+        assert rel_err(lg, out["logits"]) <= TAU[0]
+        assert nxt.shape == (B,)
+    finally:
+        fp.fp_destroy(h)
