@@ -92,6 +92,13 @@ def kernel_bytes(a, wq, kvq, B, ctx):
 # cached token row (units = B x context of the capture) and scales with the
 # bench's B x context.
 NCU_TRAFFIC = {
+    # profiles/dram_traffic_l70b.md: microbench cases 70b-*, one launch each
+    ("l70b", "lin_gu"): {"bytes": 271997952, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
+    ("l70b", "lin_down"): {"bytes": 132128000, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
+    ("l70b", "lin_qkv"): {"bytes": 45146880, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
+    ("l70b", "lin_o"): {"bytes": 36758528, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
+    ("l70b", "lm_head"): {"bytes": 535367936, "units": None, "src": "fp_linear.cu", "sha": "f7df17bc3111d3ac"},
+    ("l70b", "attn"): {"bytes": 149525504, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
     ("l7b", "attn"): {"bytes": 81739520, "units": 8 * 612, "src": "fp_attention.cu", "sha": "de945a405c820013"},
     ("l7b", "lm_head"): {"bytes": 270745088, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
     ("l7b", "lin_gu"): {"bytes": 94480640, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
@@ -365,25 +372,30 @@ def run_estimate(args, cfg):
         h = fp.fp_create(arch_dict((L,) + tuple(arch[1:])), wq, kvq, B, S + N + 1, seed=0)
         try:
             r = fp.fp_profile(h, S, n, warmup=1, iters=iters)
-            return r.request_ms, r.ttft_ms, r.tpot_ms, r.peak_hbm_bytes
+            return r.request_ms, r.ttft_ms, r.tpot_ms, r.peak_hbm_bytes, r.observed_hbm_bytes
         finally:
             fp.fp_destroy(h)
 
-    fits, mem = {}, {}
+    measure(1, lens[0], 1)  # loads every kernel once, so no reading below carries that one-time cost
+    fits, mem, obs = {}, {}, {}
     for L in (1, 2):
         lat = [measure(L, n, 3) for n in lens]
         fits[L] = fp.fp_solve_eq1(lens[0], lat[0][0], lens[1], lat[1][0])
         mem[L] = lat[0][3]
+        obs[L] = lat[1][4]
     t = fp.fp_solve_eq23(1, fits[1], 2, fits[2])
     rows = []
     for L in (3, 4, full):
-        req, ttft, tpot, peak = measure(L, N, 2)
+        req, ttft, tpot, peak, seen = measure(L, N, 2)
         pred = fp.fp_predict_latency(t, L, N)
         pmem = fp.fp_extrapolate_memory(1, mem[1], 2, mem[2], L)
+        pobs = fp.fp_extrapolate_memory(1, obs[1], 2, obs[2], L)
         rows.append({"layers": L, "output_length": N, "predicted_ms": pred, "measured_ms": req,
                      "rel_err": (pred - req) / req, "predicted_ttft_ms": L * t.ttft_layer + t.ttft_other,
                      "measured_ttft_ms": ttft, "predicted_tpot_ms": L * t.tpot_layer + t.tpot_other,
-                     "measured_tpot_ms": tpot, "predicted_peak_hbm_bytes": pmem, "measured_peak_hbm_bytes": peak})
+                     "measured_tpot_ms": tpot, "predicted_peak_hbm_bytes": pmem, "measured_peak_hbm_bytes": peak,
+                     "predicted_observed_bytes": pobs, "observed_bytes": seen,
+                     "observed_rel_err": (pobs - seen) / seen if seen else None})
     print(json.dumps({"config": config_json(args, cfg), "fits": {L: {"ttft_ms": f.ttft, "tpot_ms": f.tpot}
                                                                  for L, f in fits.items()},
                       "terms_ms": {"ttft_layer": t.ttft_layer, "ttft_other": t.ttft_other,

@@ -197,6 +197,11 @@ typedef struct fp_profile_result {
   int n_layers, prompt_len, n_decode, iters;
   double request_ms;          /* one request: prefill + n_decode decode steps, device
                                  events, mean over iters (the latency of Eq. 1) */
+  unsigned long long observed_hbm_bytes; /* device memory the deployment holds at the end
+                                 of fp_profile: free memory just before fp_create minus
+                                 free memory now (cudaMemGetInfo), the reading a monitor of
+                                 the GPU takes (Sec. 7 "Monitoring Daemon"); it counts
+                                 whatever else the process allocated in between */
 } fp_profile_result;
 
 /* Profile latency and memory, the observations the estimator consumes:

@@ -127,11 +127,12 @@ int fp_op_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, 
 size_t fp_op_attention_decode_workspace_bytes(int B, int n_heads, int head_dim, int max_len);
 
 /* Context splits fp_op_attention_decode uses for B sequences, n_kv_heads KV
- * heads and max_len cached positions (0 for a non-positive argument).  With
+ * heads of head_dim, a kvquant cache of 16-token pages with 16-byte aligned
+ * pools, and max_len cached positions (0 for a non-positive argument).  With
  * 1 split the kernel normalises in place and never touches the workspace;
  * with more, the partials go to the workspace and a second kernel merges
  * them. */
-int fp_op_attention_decode_splits(int B, int n_kv_heads, int max_len);
+int fp_op_attention_decode_splits(int B, int n_kv_heads, int head_dim, int kvquant, int max_len);
 
 /* Decode attention without a caller workspace, for callers that cannot
  * allocate device memory (a host whose device memory is all reserved by

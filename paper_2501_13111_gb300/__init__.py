@@ -76,7 +76,8 @@ class fp_profile_result(C.Structure):
                 ("weight_bytes", C.c_ulonglong), ("kv_bytes", C.c_ulonglong), ("act_bytes", C.c_ulonglong),
                 ("workspace_bytes", C.c_ulonglong), ("memgetinfo_bytes", C.c_ulonglong),
                 ("decode_bytes_per_step", C.c_ulonglong), ("n_layers", C.c_int), ("prompt_len", C.c_int),
-                ("n_decode", C.c_int), ("iters", C.c_int), ("request_ms", C.c_double)]
+                ("n_decode", C.c_int), ("iters", C.c_int), ("request_ms", C.c_double),
+                ("observed_hbm_bytes", C.c_ulonglong)]
 
     def as_dict(self):
         d = {}
@@ -141,7 +142,7 @@ _PROTOS = {
     "fp_op_rope_kv": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P, _P]),
     "fp_op_attention_decode": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _SZ, _P, _P]),
     "fp_op_attention_decode_workspace_bytes": (_SZ, [_I, _I, _I, _I]),
-    "fp_op_attention_decode_splits": (_I, [_I, _I, _I]),
+    "fp_op_attention_decode_splits": (_I, [_I, _I, _I, _I, _I]),
     "fp_op_attention_decode_noalloc": (_I, [_P, _I, _I, _I, C.POINTER(fp_kv_view), _P, _I, _P, _P, _P]),
     "fp_op_attention_prefill": (_I, [_P, _I, _I, _I, _I, C.POINTER(fp_kv_view), _P, _P, _P]),
     "fp_op_argmax": (_I, [_P, _I, _I, _P, _P]),
@@ -319,8 +320,8 @@ def fp_op_attention_decode(q, q_stride, B, n_heads, kv: fp_kv_view, lens, max_le
                                               workspace_bytes, err, stream))
 
 
-def fp_op_attention_decode_splits(B, n_kv_heads, max_len):
-    return _lib.fp_op_attention_decode_splits(B, n_kv_heads, max_len)
+def fp_op_attention_decode_splits(B, n_kv_heads, head_dim, kvquant, max_len):
+    return _lib.fp_op_attention_decode_splits(B, n_kv_heads, head_dim, kvquant, max_len)
 
 
 FP_NOALLOC_SCRATCH_BYTES = 32 << 20  # FP_NOALLOC_SCRATCH_BYTES of fp_ops.h (a CPU test keeps the two equal)

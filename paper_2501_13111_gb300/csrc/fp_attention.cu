@@ -77,10 +77,12 @@ static int dec_max_splits(long long pairs, int tiles) {
   return (int)std::max<long long>(std::max<long long>(s, 1), dec_min_splits(tiles));
 }
 
-static DecodeGeom decode_geom(int B, int n_kv_heads, int max_len) {
+// occ > 0: CTAs per SM of the kernel the geometry is for (the int8 page-streaming
+// kernel: 4); occ 0: the mma.sync tile kernel, whose ring depth sets it.
+static DecodeGeom decode_geom(int B, int n_kv_heads, int max_len, int occ = 0) {
   const long long pairs = (long long)B * n_kv_heads;
   const int nb = dec_ring_depth(pairs);
-  const long long slots = (long long)dec_sm_count() * dec_occ(nb);
+  const long long slots = (long long)dec_sm_count() * (occ > 0 ? occ : dec_occ(nb));
   const int tiles = std::max(1, (max_len + kDecTT - 1) / kDecTT);
   const int smax = std::min(dec_max_splits(pairs, tiles),
                             (int)std::max<long long>(std::min<long long>(tiles, 4), 2 * slots / std::max(1LL, pairs)));
@@ -100,12 +102,25 @@ static DecodeGeom decode_geom(int B, int n_kv_heads, int max_len) {
   return best;
 }
 
-int attention_decode_launches(int B, int n_kv_heads, int max_len) {
-  return decode_geom(B, n_kv_heads, max_len).splits == 1 ? 1 : 2;
+// The int8 cache with head_dim 128 (16-byte aligned pools, 16-token pages)
+// runs the page-streaming kernel.  It shares the tile kernel's split
+// geometry: scoring its 4 CTAs per SM split the 70B-shaped context in two,
+// which measured slower (42 us against 36 us; each warp's ring fill and the
+// merge weigh more on half the pages, and the combine pass is added).
+static bool dec_i8_shape(int kvquant, int head_dim, int page_size) {
+  return kvquant == FP_KV_INT8 && head_dim == 128 && page_size == 16;
+}
+static DecodeGeom decode_geom_for(int B, int n_kv_heads, int head_dim, int kvquant, int page_size, int max_len) {
+  (void)head_dim, (void)kvquant, (void)page_size;
+  return decode_geom(B, n_kv_heads, max_len);
 }
 
-int attention_decode_splits(int B, int n_kv_heads, int max_len) {
-  return decode_geom(B, n_kv_heads, max_len).splits;
+int attention_decode_launches(int B, int n_kv_heads, int head_dim, int kvquant, int max_len) {
+  return decode_geom_for(B, n_kv_heads, head_dim, kvquant, 16, max_len).splits == 1 ? 1 : 2;
+}
+
+int attention_decode_splits(int B, int n_kv_heads, int head_dim, int kvquant, int max_len) {
+  return decode_geom_for(B, n_kv_heads, head_dim, kvquant, 16, max_len).splits;
 }
 
 size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len) {
@@ -832,11 +847,11 @@ static cudaError_t launch_decode_g(int G, const uint16_t* q, int q_stride, int B
 cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, const fp_kv_view& kv,
                                     const int32_t* len, int len_add, int max_len, uint16_t* out, void* ws,
                                     int32_t* err, cudaStream_t s, cudaError_t* second) {
-  DecodeGeom g = decode_geom(B, kv.n_kv_heads, max_len);
   const int G = n_heads / kv.n_kv_heads;
   float* w = (float*)ws;
   const bool a16 = (((uintptr_t)kv.k_pool | (uintptr_t)kv.v_pool | (uintptr_t)kv.k_scale | (uintptr_t)kv.v_scale) & 15) == 0;
-  if (kv.kvquant == FP_KV_INT8 && kv.head_dim == 128 && kv.page_size == 16 && a16) {
+  if (dec_i8_shape(kv.kvquant, kv.head_dim, kv.page_size) && a16) {
+    const DecodeGeom g = decode_geom_for(B, kv.n_kv_heads, kv.head_dim, kv.kvquant, kv.page_size, max_len);
     switch (G) {
       case 1: return launch_decode_i8<1>(q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second);
       case 2: return launch_decode_i8<2>(q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second);
@@ -845,6 +860,7 @@ cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int 
       default: return cudaErrorInvalidValue;
     }
   }
+  const DecodeGeom g = decode_geom(B, kv.n_kv_heads, max_len);
   if (kv.head_dim == 64) {
     return kv.kvquant == FP_KV_BF16
                ? launch_decode_g<64, FP_KV_BF16>(G, q, q_stride, B, n_heads, kv, len, len_add, max_len, g, w, out, err, s, second)

@@ -48,11 +48,14 @@ constexpr uint32_t kTcTmemCols = 512;  // two 256-column fp32 accumulators
 // and weight columns stay in L2).  The shared ring runs across tiles, and
 // the fp32 accumulator is double-buffered in TMEM (2 x 256 columns): the MMA
 // thread fills one buffer while the epilogue warps drain the other.
-// SCALE: multiply output column n by bf16 scales[n] (int8 weights).
+// SCALE: multiply output column n by bf16 scales[n] (int8 weights; SwiGLU:
+// the up column by scales[up_off + n]).  Output (and residual) rows are ldy
+// elements apart, so a launch can fill a band of columns of a wider output.
 template <int EPI, bool SCALE>
 __global__ void __launch_bounds__(kTcThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap map_x, const __grid_constant__ CUtensorMap map_w, int M, int N,
-                   int K, const uint16_t* __restrict__ scales, const uint16_t* R, void* Y, int32_t* err) {
+                   int K, const uint16_t* __restrict__ scales, long long up_off, const uint16_t* R, void* Y,
+                   int ldy, int32_t* err) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   __shared__ uint64_t full[kTcStages], empty[kTcStages], tfull[2], tempty[2], mma_done;
   __shared__ uint32_t tmem_base;
@@ -205,11 +208,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           for (int i = 0; i < 32; ++i) {
             if (i < cnt) {
               v[i] *= bf2f(scales[n + i]);
-              if (NR == 2) u[i] *= bf2f(scales[Nout + n + i]);
+              if (NR == 2) u[i] *= bf2f(scales[up_off + n + i]);
             }
           }
         }
-        const long long o = (long long)row * Nout + n;
+        const long long o = (long long)row * ldy + n;
         if constexpr (EPI == FP_EPI_F32) {
           float* y = (float*)Y + o;
           if (cnt == 32 && (o & 3) == 0) {
@@ -330,13 +333,33 @@ static bool make_map(CUtensorMap* map, const void* base, long long rows, long lo
   return make_tensor_map(map, base, rows, cols, 2, box_rows, kTcBK, 128);
 }
 
-size_t gemm_tc_ws_bytes(int wquant, int N, int K) { return wquant == FP_W_BF16 ? 0 : (size_t)N * K * 2; }
+// Quantised weights are expanded to bf16 band by band of output columns, so
+// the scratch holds at most kTcScratchBytes (or one band of 256 columns).
+constexpr size_t kTcScratchBytes = 128u << 20;
+
+// Output columns per band: a multiple of the tile's (256, SwiGLU 128), all of them if they fit.
+static int band_cols(int epi, int N, int K) {
+  const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
+  const int nout = nr == 2 ? N / 2 : N;
+  const int unit = kTcBN / nr;
+  const long long fit = (long long)(kTcScratchBytes / ((size_t)nr * K * 2)) / unit * unit;
+  return (int)std::min<long long>(nout, std::max<long long>(unit, fit));
+}
+
+size_t gemm_tc_ws_bytes(int wquant, int N, int K) {
+  if (wquant == FP_W_BF16) return 0;
+  // the largest band over the epilogues (a SwiGLU band holds its gate and its up rows)
+  const size_t plain = (size_t)band_cols(FP_EPI_STORE, N, K) * K * 2;
+  const size_t swiglu = N % 2 == 0 ? (size_t)2 * band_cols(FP_EPI_SWIGLU, N, K) * K * 2 : 0;
+  return std::max(plain, swiglu);
+}
 
 bool gemm_tc_ok(int M, int N, int K) { return M > 64 && K % 8 == 0 && N >= 1 && encode_fn() != nullptr; }
 
 template <int EPI, bool SCALE>
 static cudaError_t launch_tc_t(const CUtensorMap& mx, const CUtensorMap& mw, int M, int N, int K,
-                               const uint16_t* scales, const uint16_t* R, void* Y, int32_t* err, cudaStream_t s) {
+                               const uint16_t* scales, long long up_off, const uint16_t* R, void* Y, int ldy,
+                               int32_t* err, cudaStream_t s) {
   auto kern = gemm_tc_kernel<EPI, SCALE>;
   const size_t smem = (size_t)kTcStages * kTcStageBytes + 1024;
   static std::atomic<unsigned long long> attr{0};
@@ -353,38 +376,67 @@ static cudaError_t launch_tc_t(const CUtensorMap& mx, const CUtensorMap& mw, int
   }
   // persistent: one CTA per SM (its shared ring and 512 TMEM columns fill the SM)
   const dim3 grid((unsigned)std::min<long long>(tiles, sms));
-  return launch(kern, grid, dim3(kTcThreads), smem, s, mx, mw, M, N, K, scales, R, Y, err);
+  return launch(kern, grid, dim3(kTcThreads), smem, s, mx, mw, M, N, K, scales, up_off, R, Y, ldy, err);
+}
+
+template <int EPI>
+static cudaError_t launch_tc_e(bool sc, const CUtensorMap& mx, const CUtensorMap& mw, int M, int N, int K,
+                               const uint16_t* scales, long long up_off, const uint16_t* R, void* Y, int ldy,
+                               int32_t* err, cudaStream_t s) {
+  return sc ? launch_tc_t<EPI, true>(mx, mw, M, N, K, scales, up_off, R, Y, ldy, err, s)
+            : launch_tc_t<EPI, false>(mx, mw, M, N, K, scales, up_off, R, Y, ldy, err, s);
+}
+
+static cudaError_t launch_tc_any(int epi, bool sc, const CUtensorMap& mx, const CUtensorMap& mw, int M, int N, int K,
+                                 const uint16_t* scales, long long up_off, const uint16_t* R, void* Y, int ldy,
+                                 int32_t* err, cudaStream_t s) {
+  switch (epi) {
+    case FP_EPI_STORE: return launch_tc_e<FP_EPI_STORE>(sc, mx, mw, M, N, K, scales, up_off, R, Y, ldy, err, s);
+    case FP_EPI_RESID: return launch_tc_e<FP_EPI_RESID>(sc, mx, mw, M, N, K, scales, up_off, R, Y, ldy, err, s);
+    case FP_EPI_SWIGLU: return launch_tc_e<FP_EPI_SWIGLU>(sc, mx, mw, M, N, K, scales, up_off, R, Y, ldy, err, s);
+    default: return launch_tc_e<FP_EPI_F32>(sc, mx, mw, M, N, K, scales, up_off, R, Y, ldy, err, s);
+  }
+}
+
+// Expand rows [r0, r0 + rows) of a quantised matrix into out [rows][K] bf16.
+static cudaError_t dequant_rows(int wquant, const void* codes, const uint16_t* scales, const uint16_t* zeros, long long r0,
+                                int rows, int K, uint16_t* out, cudaStream_t s) {
+  const uint8_t* c = (const uint8_t*)codes + (wquant == FP_W_INT8 ? r0 * K : r0 * (K / 2));
+  const uint16_t* sc = wquant == FP_W_INT4_G128 ? scales + r0 * (K / 128) : scales;
+  const uint16_t* ze = wquant == FP_W_INT4_G128 ? zeros + r0 * (K / 128) : zeros;
+  const long long words = (long long)rows * K / 8;
+  const int blocks = (int)std::min<long long>((words + 255) / 256, 152 * 16);
+  return launch(dequant_kernel, dim3(blocks), dim3(256), 0, s, wquant, (const void*)c, sc, ze, rows, K, out);
 }
 
 cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                            const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
                            void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s) {
-  const uint16_t* w = (const uint16_t*)codes;
-  if (wquant != FP_W_BF16) {
-    if (!ws || ws_bytes < gemm_tc_ws_bytes(wquant, N, K)) return cudaErrorInvalidValue;
-    const long long words = (long long)N * K / 8;
-    const int blocks = (int)std::min<long long>((words + 255) / 256, 152 * 16);
-    FP_CUDA_TRY(launch(dequant_kernel, dim3(blocks), dim3(256), 0, s, wquant, codes, scales, zeros, N, K, (uint16_t*)ws));
-    w = (const uint16_t*)ws;
-  }
-  CUtensorMap mx, mw;
+  const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
+  const int Nout = nr == 2 ? N / 2 : N;
   const int wbox = epi == FP_EPI_SWIGLU ? 128 : 256;
-  if (!make_map(&mx, x, M, K, kTcBM) || !make_map(&mw, w, N, K, wbox)) return cudaErrorInvalidValue;
   const bool sc = wquant == FP_W_INT8;
-  switch (epi) {
-    case FP_EPI_STORE:
-      return sc ? launch_tc_t<FP_EPI_STORE, true>(mx, mw, M, N, K, scales, residual, y, err, s)
-                : launch_tc_t<FP_EPI_STORE, false>(mx, mw, M, N, K, scales, residual, y, err, s);
-    case FP_EPI_RESID:
-      return sc ? launch_tc_t<FP_EPI_RESID, true>(mx, mw, M, N, K, scales, residual, y, err, s)
-                : launch_tc_t<FP_EPI_RESID, false>(mx, mw, M, N, K, scales, residual, y, err, s);
-    case FP_EPI_SWIGLU:
-      return sc ? launch_tc_t<FP_EPI_SWIGLU, true>(mx, mw, M, N, K, scales, residual, y, err, s)
-                : launch_tc_t<FP_EPI_SWIGLU, false>(mx, mw, M, N, K, scales, residual, y, err, s);
-    default:
-      return sc ? launch_tc_t<FP_EPI_F32, true>(mx, mw, M, N, K, scales, residual, y, err, s)
-                : launch_tc_t<FP_EPI_F32, false>(mx, mw, M, N, K, scales, residual, y, err, s);
+  CUtensorMap mx, mw;
+  if (!make_map(&mx, x, M, K, kTcBM)) return cudaErrorInvalidValue;
+  if (wquant == FP_W_BF16) {
+    if (!make_map(&mw, codes, N, K, wbox)) return cudaErrorInvalidValue;
+    return launch_tc_any(epi, sc, mx, mw, M, N, K, scales, Nout, residual, y, Nout, err, s);
   }
+  if (!ws || ws_bytes < gemm_tc_ws_bytes(wquant, N, K)) return cudaErrorInvalidValue;
+  // band by band of output columns: expand the band's rows (SwiGLU: its gate
+  // rows, then its up rows) into the scratch, then multiply
+  uint16_t* w = (uint16_t*)ws;
+  const int band = band_cols(epi, N, K);
+  for (int c0 = 0; c0 < Nout; c0 += band) {
+    const int cols = std::min(band, Nout - c0);
+    FP_CUDA_TRY(dequant_rows(wquant, codes, scales, zeros, c0, cols, K, w, s));
+    if (nr == 2) FP_CUDA_TRY(dequant_rows(wquant, codes, scales, zeros, (long long)Nout + c0, cols, K, w + (size_t)cols * K, s));
+    if (!make_map(&mw, w, (long long)nr * cols, K, wbox)) return cudaErrorInvalidValue;
+    const uint16_t* r = residual ? residual + c0 : nullptr;
+    void* yb = epi == FP_EPI_F32 ? (void*)((float*)y + c0) : (void*)((uint16_t*)y + c0);
+    FP_CUDA_TRY(launch_tc_any(epi, sc, mx, mw, M, nr * cols, K, sc ? scales + c0 : scales, Nout, r, yb, Nout, err, s));
+  }
+  return cudaSuccess;
 }
 
 }  // namespace fpk

@@ -114,9 +114,9 @@ size_t fp_op_attention_decode_workspace_bytes(int B, int n_heads, int head_dim, 
   return attention_decode_ws_bytes(B, n_heads, head_dim, max_len);
 }
 
-int fp_op_attention_decode_splits(int B, int n_kv_heads, int max_len) {
-  if (B <= 0 || n_kv_heads <= 0 || max_len <= 0) return 0;
-  return attention_decode_splits(B, n_kv_heads, max_len);
+int fp_op_attention_decode_splits(int B, int n_kv_heads, int head_dim, int kvquant, int max_len) {
+  if (B <= 0 || n_kv_heads <= 0 || head_dim <= 0 || max_len <= 0) return 0;
+  return attention_decode_splits(B, n_kv_heads, head_dim, kvquant, max_len);
 }
 
 static bool group_ok(int n_heads, int n_kv_heads) {

@@ -102,6 +102,7 @@ struct fp_handle {
   void* arena = nullptr;
   size_t arena_bytes = 0;
   unsigned long long weight_bytes = 0, kv_bytes = 0, act_bytes = 0, ws_bytes = 0, memgetinfo_bytes = 0;
+  size_t free_before = 0;  // free device memory just before fp_create reserved anything
 
   uint16_t *embed = nullptr, *final_norm = nullptr, *lm_head = nullptr;
   Layer L[FP_MAX_LAYERS];
@@ -303,7 +304,7 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
                                               h->attn_ws, h->err, s, &e2);
       if (e != cudaSuccess) return h->cuda_fail(e, "attention decode");
       // the split kernel and the combine kernel (when there is one) are timed together
-      h->launches += attention_decode_launches(B, a.n_kv_heads, h->T);
+      h->launches += attention_decode_launches(B, a.n_kv_heads, a.head_dim, h->kvq, h->T);
       h->tr.after(FP_K_ATTN);
     } else {
       LTRY(launch_attention_prefill(h->qkv, h->n_qkv, B, S, a.n_heads, kv, h->att, h->err, s), FP_K_ATTN);
@@ -534,6 +535,7 @@ int fp_create(const fp_arch* arch, int wquant, int kvquant, int batch, int max_c
   }
   cudaMemGetInfo(&free1, &total);
   h->memgetinfo_bytes = free0 > free1 ? free0 - free1 : 0;
+  h->free_before = free0;
   carve(h, (char*)h->arena);
 
   e = cudaMemsetAsync(h->arena, 0, h->arena_bytes, h->stream);
@@ -919,6 +921,13 @@ int fp_profile(fp_handle* h, int prompt_len, int n_decode, int warmup, int iters
       out->kernel_ms[k] = kms[k] / ksteps;
       out->kernel_launches[k] = kl[k];
     }
+  }
+  // observed: the device memory the deployment holds now, after its passes
+  // (arena, decode graph, loaded kernels), as a monitor of the GPU sees it
+  {
+    size_t free_now = 0, total = 0;
+    if (cudaMemGetInfo(&free_now, &total) == cudaSuccess && h->free_before > free_now)
+      out->observed_hbm_bytes = h->free_before - free_now;
   }
   return check_err_flag(h);
 }

@@ -33,9 +33,9 @@ cudaError_t launch_rope_kv(uint16_t* qkv, int B, int S, int row_stride, int n_he
 // ---- attention (fp_attention.cu)
 size_t attention_decode_ws_bytes(int B, int n_heads, int head_dim, int max_len);
 // Kernels one decode-attention launch runs: 1 (one split, normalised in place) or 2 (splits + combine).
-int attention_decode_launches(int B, int n_kv_heads, int max_len);
+int attention_decode_launches(int B, int n_kv_heads, int head_dim, int kvquant, int max_len);
 // Context splits of one decode-attention launch (1: the partials workspace is not touched).
-int attention_decode_splits(int B, int n_kv_heads, int max_len);
+int attention_decode_splits(int B, int n_kv_heads, int head_dim, int kvquant, int max_len);
 cudaError_t launch_attention_decode(const uint16_t* q, int q_stride, int B, int n_heads, const fp_kv_view& kv,
                                     const int32_t* len, int len_add, int max_len, uint16_t* out, void* ws,
                                     int32_t* err, cudaStream_t s, cudaError_t* second = nullptr);

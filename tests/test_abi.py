@@ -205,6 +205,8 @@ def test_binding_constants_match_the_headers(fp):
 def test_decode_splits_query_answers_on_host(fp):
     """The split count is host arithmetic (no GPU call): one split for a short
     context, several for the 70B-shaped decode attention."""
-    assert fp.fp_op_attention_decode_splits(0, 8, 100) == 0
-    assert fp.fp_op_attention_decode_splits(1, 1, 10) == 1
-    assert fp.fp_op_attention_decode_splits(2, 8, 2155) > 1
+    assert fp.fp_op_attention_decode_splits(0, 8, 128, 1, 100) == 0
+    assert fp.fp_op_attention_decode_splits(1, 1, 128, 0, 10) == 1
+    assert fp.fp_op_attention_decode_splits(2, 8, 128, 1, 2155) > 1
+    # the 70B-shaped decode: 256 (sequence, KV head) pairs fill the GPU, one split
+    assert fp.fp_op_attention_decode_splits(32, 8, 128, 1, 2149) == 1

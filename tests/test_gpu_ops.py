@@ -430,3 +430,32 @@ def test_prefill_gemm_matches_oracle(fp, wq, epi, m, n, k):
         else:
             ref = M.silu(yref[:, :nout]) * yref[:, nout:]
     assert rel_err(got, ref) <= TAU[wq] / 4, (wq, epi, m, n, k, rel_err(got, ref))
+
+
+@pytest.mark.parametrize("wq,m,n,k,epi", [(1, 200, 2 * 9000, 8192, 2), (2, 136, 20000, 4096, 1), (1, 130, 17000, 4096, 3)])
+def test_prefill_linear_in_bands_of_columns(fp, wq, m, n, k, epi):
+    """Quantised prefill weights are expanded to bf16 band by band of output
+    columns (the scratch holds at most 128 MB): matrices larger than that run
+    as several expansions and GEMM launches into slices of the output.  Cases:
+    int8 SwiGLU (up rows' scales taken at an offset, 3 bands of 4096 + 808
+    columns), int4 with residual (2 bands), int8 fp32 out (2 bands)."""
+    w = synth.weight_bf16(70 + wq, 0, 1, (n, k))
+    x = synth.uniform_bf16(71, m, (m, k), -2.0, 2.0)
+    nout = n // 2 if epi == 2 else n
+    r = synth.uniform_bf16(72, m, (m, nout), -1.0, 1.0)
+    codes, scales, zeros = _quantized_on_device(fp, wq, w)
+    _, wd = quant.quantize_weight(w, wq)
+    assert fp.fp_op_linear_workspace_bytes(wq, m, n, k) <= (128 << 20) + (1 << 20)
+    out = empty(m * nout * (4 if epi == 3 else 2))
+    ws_b = fp.fp_op_linear_workspace_bytes(wq, m, n, k)
+    ws = empty(max(ws_b, 16))
+    fp.fp_op_linear(wq, epi, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(dev(r)), ptr(out),
+                    ptr(ws), ws_b)
+    got = host(out, np.float32) if epi == 3 else quant.bf16_to_f32(host(out, np.uint16))
+    got = got.reshape(m, nout).astype(np.float64)
+    y = quant.bf16_to_f32(x).astype(np.float64) @ wd.T
+    if epi == 1:
+        y = quant.bf16_to_f32(r).astype(np.float64) + y
+    elif epi == 2:
+        y = M.silu(y[:, :nout]) * y[:, nout:]
+    assert rel_err(got, y) <= TAU[wq] / 4, rel_err(got, y)

@@ -40,7 +40,7 @@ def _paged_cache(fp, kvq, B, T, Hkv, hd, seed):
 def _both(fp, kvq, lens, H, Hkv, hd, seed):
     """(allocating result, no-allocation result, error words) for one shape."""
     B, T = len(lens), max(lens) + 7
-    assert fp.fp_op_attention_decode_splits(B, Hkv, T) > 1, "the case must use the split partials"
+    assert fp.fp_op_attention_decode_splits(B, Hkv, hd, kvq, T) > 1, "the case must use the split partials"
     kv = _paged_cache(fp, kvq, B, T, Hkv, hd, seed)
     q = dev(synth.uniform_bf16(seed, 3, (B, H * hd), -2, 2))
     ln = dev(np.array(lens, np.int32))
