@@ -62,9 +62,16 @@ enum {
  * 17 <= M <= 64 and 16-byte aligned x and codes, which runs on tcgen05 with
  * each weight expanded to bf16((q - z) s) as the prefill GEMM does; a K that
  * is not a multiple of the GEMV's K step falls back to one warp per output
- * row on the CUDA cores -- larger M the tcgen05 GEMM.  workspace: 16-byte aligned, at least
+ * row on the CUDA cores -- larger M the tcgen05 GEMM.  For M > 64 with int8
+ * or int4 weights the GEMM either reads a bf16 expansion of W that it writes
+ * into the workspace band by band (at most 128 MB; the faster path), or, when
+ * the workspace is NULL or smaller than that, dequantises the codes inside
+ * the GEMM (bf16 weight tiles built in shared memory for every 256-token
+ * tile; no workspace; about two thirds of the speed; x and codes 16-byte
+ * aligned).  workspace: 16-byte aligned, at least
  * fp_op_linear_workspace_bytes(wquant, M, N, K) bytes (may be NULL when that
- * is 0), else FP_ERR_INVALID_ARG.  Its leading bytes are ticket counters
+ * is 0, or for the in-kernel dequantisation above), else FP_ERR_INVALID_ARG.
+ * Its leading bytes are ticket counters
  * that must be zero before the first call (e.g. a zeroed buffer); every call
  * leaves them zero again, so one workspace serves any sequence of calls on
  * one stream (calls that overlap on the GPU need separate workspaces). */

@@ -824,6 +824,9 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (M > 64 && gemm_tc_ok(M, N, K)) {
     const size_t need = linear_ws_bytes(wquant, M, N, K);
+    // int8 / int4 without room for the bf16 expansion: dequantise inside the GEMM
+    if (need > 0 && (!ws || ws_bytes < need) && gemm_wq_ok(wquant, epi, M, N, K, x, codes))
+      return launch_gemm_wq(wquant, epi, x, M, N, K, codes, scales, zeros, residual, y, err, s);
     if (need > 0 && (!ws || ws_bytes < need)) return cudaErrorInvalidValue;
     void* scratch = need ? (char*)ws + counter_bytes(0) : nullptr;
     return launch_gemm_tc(wquant, epi, x, M, N, K, codes, scales, zeros, residual, y, scratch,

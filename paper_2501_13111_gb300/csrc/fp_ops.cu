@@ -61,7 +61,11 @@ int fp_op_linear(int wquant, int epilogue, const uint16_t* x, int M, int N, int 
   if (K % k_align(wquant) != 0) return FP_ERR_UNSUPPORTED;
   if (M == 0) return FP_OK;
   size_t need = linear_ws_bytes(wquant, M, N, K);
-  if (need > 0 && (!workspace || workspace_bytes < need)) return FP_ERR_INVALID_ARG;
+  // quantised prefill without room for the bf16 expansion: the GEMM that
+  // dequantises in the kernel needs no workspace
+  const bool no_scratch = !workspace || workspace_bytes < need;
+  const bool in_kernel = M > 64 && wquant != FP_W_BF16 && no_scratch && gemm_wq_ok(wquant, epilogue, M, N, K, x, codes);
+  if (need > 0 && no_scratch && !in_kernel) return FP_ERR_INVALID_ARG;
   return cuda_status(launch_linear(wquant, epilogue, x, M, N, K, codes, scales, zeros, residual, y, workspace,
                                    workspace_bytes, (cudaStream_t)stream));
 }

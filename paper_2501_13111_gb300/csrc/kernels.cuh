@@ -71,4 +71,10 @@ cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N,
                            const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
                            void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s);
 
+// ---- prefill GEMM with int8 / int4 weights dequantised in the kernel (fp_gemm_wq.cu)
+bool gemm_wq_ok(int wquant, int epi, int M, int N, int K, const void* x, const void* codes);
+cudaError_t launch_gemm_wq(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
+                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                           int32_t* err, cudaStream_t s);
+
 }  // namespace fpk

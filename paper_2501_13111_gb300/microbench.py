@@ -13,7 +13,8 @@ calls, which is the shape a profiler capture wants (``-s 2 -c 1``).
 
 Decode linears report GB/s of algorithmic bytes (codes + scales/zeros +
 activations in and out); attention reports GB/s of cached K/V (+ int8 scales);
-the prefill GEMM reports TFLOP/s of 2·M·N·K and prefill attention those of
+the prefill GEMM reports TFLOP/s of 2·M·N·K (``-inkernel`` cases: int8 / int4
+weights dequantised inside the GEMM, no workspace) and prefill attention those of
 both matmuls over the causal half, 2·B·H·S²·hd.  Weights and caches hold random
 values: speed does not depend on them.
 """
@@ -61,7 +62,7 @@ def quantized(wq, n, k):
     return codes, sc, ze
 
 
-def case_linear(wq, epi, M, N, K, single, iters):
+def case_linear(wq, epi, M, N, K, scratch=True, *, single, iters):
     nbytes = weight_bytes(N, K, wq)
     copies = 1 if single else max(2, min(8, -(-3 * L2_BYTES // nbytes)))
     mats = [quantized(wq, N, K) for _ in range(copies)]
@@ -69,13 +70,14 @@ def case_linear(wq, epi, M, N, K, single, iters):
     nout = N // 2 if epi == 2 else N
     y = torch.zeros(M * nout * 4, dtype=torch.uint8, device="cuda")
     r = torch.zeros(M * nout, dtype=torch.bfloat16, device="cuda")
-    wsb = fp.fp_op_linear_workspace_bytes(wq, M, N, K)
+    wsb = fp.fp_op_linear_workspace_bytes(wq, M, N, K) if scratch else 0
     ws = torch.zeros(max(wsb, 16), dtype=torch.uint8, device="cuda")
+    wsp = ws.data_ptr() if scratch else None
 
     def f():
         for codes, sc, ze in mats:
             fp.fp_op_linear(wq, epi, x.data_ptr(), M, N, K, codes.data_ptr(), sc.data_ptr(), ze.data_ptr(),
-                            r.data_ptr(), y.data_ptr(), ws.data_ptr(), wsb)
+                            r.data_ptr(), y.data_ptr(), wsp, wsb)
 
     ms = timed(f, iters) / copies
     out_elt = 4 if epi == 3 else 2
@@ -185,7 +187,14 @@ CASES["7b-qkv-prefill"] = ("linear", (1, 0, 4096, 12288, 4096))
 CASES["7b-gu-prefill"] = ("linear", (1, 2, 4096, 22016, 4096))
 CASES["7b-down-prefill"] = ("linear", (1, 1, 4096, 4096, 11008))
 CASES["13b-gu-prefill"] = ("linear", (2, 2, 16384, 27648, 5120))
+CASES["70b-qkv-prefill"] = ("linear", (2, 0, 65536, 10240, 8192))
+CASES["70b-gu-prefill"] = ("linear", (2, 2, 65536, 57344, 8192))
+CASES["70b-down-prefill"] = ("linear", (2, 1, 65536, 8192, 28672))
 CASES["bf16-8k-prefill"] = ("linear", (0, 0, 8192, 8192, 8192))
+# the same quantised prefill linears without a workspace: dequantised inside the GEMM
+for _name in ["7b-qkv-prefill", "7b-gu-prefill", "7b-down-prefill", "13b-gu-prefill", "70b-qkv-prefill",
+              "70b-gu-prefill", "70b-down-prefill"]:
+    CASES[_name + "-inkernel"] = ("linear", CASES[_name][1] + (False,))
 
 RUNNERS = {"linear": case_linear, "attention": case_attention, "attention_prefill": case_attention_prefill,
            "argmax": case_argmax}
