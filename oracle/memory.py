@@ -9,6 +9,7 @@ exact byte counts of the storage formats read in ``quant.py``:
     bf16 matrix [N, K]:  2 N K
     int8 matrix:         N K + 2 N              (codes + bf16 scale per row)
     int4 matrix:         N K / 2 + 4 N K / 128  (packed codes + bf16 scale and zero per group)
+    GPTQ4 matrix:        the int4 bytes + 4 K   (+ the int32 act order of the K input channels)
     KV per token per block: bf16 2 * Hkv * hd * 2;  int8 2 * Hkv * hd + 2 * Hkv * 4 (fp32 scales)
 
 Decode reads every block matrix, the K/V of every cached token and the LM
@@ -24,6 +25,8 @@ def matrix_bytes(n: int, k: int, wquant: int) -> int:
         return n * k + 2 * n
     if wquant == 2:
         return n * k // 2 + 4 * n * (k // 128)
+    if wquant == 3:
+        return n * k // 2 + 4 * n * (k // 128) + 4 * k
     raise ValueError(wquant)
 
 

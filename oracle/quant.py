@@ -23,6 +23,17 @@ int4 weights, asymmetric, groups of 128 along K (row n, group g):
     element NIBBLE_ORDER[i] = (0, 2, 4, 6, 1, 3, 5, 7).  So the nibble pair
     (i, i + 4) -- the pair a mask of 0x000F000F selects -- is (e_2i, e_2i+1).
 
+GPTQ-format int4 with act order (GPTQ4 in the table "Models and
+configurations"; Sec. 3.2), read as int4 group-128 over groups formed in an
+act order: a permutation perm of the K input channels; group g holds the
+channels perm[128 g .. 128 g + 127], i.e. channel k is in group
+g_idx[k] = (position of k in perm) // 128.  No calibration data exists here,
+so the codes are rounded to nearest with the int4 rule above applied to each
+group's values (GPTQ's error feedback needs calibration activations).
+    dequantised weight W[n, k] = (q[n, k] - z[n, g_idx[k]]) * s[n, g_idx[k]]
+    Storage: codes in act order (column j of the packed matrix is channel
+    perm[j]), packed as int4 above; scales and zeros [N, K/128] per group.
+
 int8 KV cache, per token and per KV head, separately for K (after RoPE) and V:
     s = fp32(max |x| / 127) (stored as fp32), q = clamp(rint(fp32(x / s)), -127, 127)
     dequantised value = q * s;  s = 0 gives q = 0.
@@ -130,6 +141,42 @@ def dequant_int4(packed, scale_bits, zero_bits) -> np.ndarray:
     return ((q - z[..., None]) * s[..., None]).reshape(n, k)
 
 
+# ---------------------------------------------------------------- GPTQ4 (act order)
+def g_idx_of(perm: np.ndarray) -> np.ndarray:
+    """Group of every input channel: g_idx[perm[j]] = j // 128."""
+    perm = np.asarray(perm, dtype=np.int64)
+    g = np.empty(perm.shape[0], dtype=np.int64)
+    g[perm] = np.arange(perm.shape[0]) // GROUP
+    return g
+
+
+def quantize_gptq4(w_bits: np.ndarray, perm: np.ndarray):
+    """int4 over act-order groups.  w_bits: bf16 bits [N, K], perm: a
+    permutation of range(K).  Returns (packed codes in act order [N, K/2],
+    scale bits [N, K/128], zero bits [N, K/128]): the int4 rule on each
+    group's values w[:, perm[128 g:128 g + 128]]."""
+    perm = np.asarray(perm, dtype=np.int64)
+    assert sorted(perm.tolist()) == list(range(w_bits.shape[1]))
+    return quantize_int4_g128(np.ascontiguousarray(w_bits[:, perm]))
+
+
+def codes_gptq4(packed: np.ndarray, perm: np.ndarray) -> np.ndarray:
+    """Codes q[n, k] in channel order from the act-order storage."""
+    qa = unpack_int4(packed)
+    q = np.empty_like(qa)
+    q[:, np.asarray(perm, dtype=np.int64)] = qa
+    return q
+
+
+def dequant_gptq4(packed, scale_bits, zero_bits, perm) -> np.ndarray:
+    """W[n, k] = (q[n, k] - z[n, g_idx[k]]) * s[n, g_idx[k]] (channel order)."""
+    q = codes_gptq4(packed, perm).astype(np.float64)
+    g = g_idx_of(perm)
+    s = bf16_to_f32(scale_bits).astype(np.float64)[:, g]
+    z = bf16_to_f32(zero_bits).astype(np.float64)[:, g]
+    return (q - z) * s
+
+
 # ---------------------------------------------------------------- int8 KV cache
 def quantize_kv_int8(x_bits: np.ndarray):
     """Per-row (token, KV head) absmax int8 quantiser over the last axis.
@@ -150,11 +197,16 @@ def dequant_kv_int8(codes: np.ndarray, scales: np.ndarray) -> np.ndarray:
 
 
 # ---------------------------------------------------------------- one entry point
-def quantize_weight(w_bits: np.ndarray, wquant: int):
-    """wquant 0 = bf16 (no codes), 1 = int8 per channel, 2 = int4 group 128.
+def quantize_weight(w_bits: np.ndarray, wquant: int, perm=None):
+    """wquant 0 = bf16 (no codes), 1 = int8 per channel, 2 = int4 group 128,
+    3 = GPTQ4 (int4 over the act order perm).
 
     Returns (payload dict, dequantised fp64 matrix).
     """
+    if wquant == 3:
+        p, s, z = quantize_gptq4(w_bits, perm)
+        return {"codes": p, "scales": s, "zeros": z, "perm": np.asarray(perm, dtype=np.int32)}, \
+            dequant_gptq4(p, s, z, perm)
     if wquant == 0:
         return {"w": w_bits}, bf16_to_f32(w_bits).astype(np.float64)
     if wquant == 1:

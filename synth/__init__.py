@@ -20,6 +20,11 @@ in ``paper_2501_13111_gb300/csrc/fp_quant.cu`` and ``common.cuh``):
   so host and device produce bit-identical weights.
 * Token ids: Lemire's multiply-shift maps the high 32 bits of a draw onto
   ``[0, vocab)``.
+* Act orders (the input-channel permutation of a GPTQ-format matrix): the
+  Fisher-Yates shuffle in Durstenfeld's form over the identity, for
+  ``i = K-1 .. 1`` swapping entry ``i`` with entry ``j``, ``j`` the
+  multiply-shift of draw ``K-1-i`` onto ``[0, i]``.  The runtime draws the
+  same permutation on the host (``csrc/fp_runtime.cu``).
 """
 from __future__ import annotations
 
@@ -44,6 +49,12 @@ TOKEN_STREAM = 1 << 20
 
 def weight_stream(layer: int, tensor: int) -> int:
     return (layer + 1) * 16 + tensor
+
+
+def perm_stream(layer: int, mat: int) -> int:
+    """Stream of the act order of fused matrix ``mat`` (0 QKV, 1 O, 2 gate+up,
+    3 down) of block ``layer``: slots 9..12 of the layer's 16 streams."""
+    return (layer + 1) * 16 + 9 + mat
 
 
 def _mix64_int(z: int) -> int:
@@ -145,3 +156,16 @@ def uniform_f32(seed: int, stream: int, shape, lo: float, hi: float) -> np.ndarr
     n = int(np.prod(shape))
     u = (draws(seed, stream, 0, n) >> np.uint64(11)).astype(np.float64) * (1.0 / (1 << 53))
     return (lo + (hi - lo) * u).astype(np.float32).reshape(shape)
+
+
+def act_order(seed: int, layer: int, mat: int, k: int) -> np.ndarray:
+    """The seeded act order of one matrix: a permutation of 0 .. k-1 (int32)."""
+    p = np.arange(k, dtype=np.int64)
+    if k < 2:
+        return p.astype(np.int32)
+    hi = draws(seed, perm_stream(layer, mat), 0, k - 1) >> np.uint64(32)
+    for t in range(k - 1):
+        i = k - 1 - t
+        j = int((int(hi[t]) * (i + 1)) >> 32)
+        p[i], p[j] = p[j], p[i]
+    return p.astype(np.int32)

@@ -17,17 +17,20 @@ L7 = Arch(2, 4096, 32, 32, 128, 11008, 32000)
 L70 = Arch(2, 8192, 64, 8, 128, 28672, 32000)
 
 
-@pytest.mark.parametrize("wq", [0, 1, 2])
+@pytest.mark.parametrize("wq", [0, 1, 2, 3])
 def test_matrix_bytes_match_quantiser_output(wq):
     w = synth.weight_bf16(0, 0, 1, (6, 384))
-    payload, _ = quant.quantize_weight(w, wq)
+    payload, _ = quant.quantize_weight(w, wq, synth.act_order(0, 0, 0, 384) if wq == 3 else None)
     assert sum(a.nbytes for a in payload.values()) == memory.matrix_bytes(6, 384, wq)
 
 
 def test_quantisation_memory_ratios_match_paper():
+    """INT8 halves and INT4 quarters the weight memory; GPTQ4 cuts it by about
+    75 % too (Sec. 3.2 "Effect of Quantization")."""
     bf16 = memory.block_weight_bytes(L70, 0)
     assert abs(memory.block_weight_bytes(L70, 1) / bf16 - 0.50) < 0.01
     assert abs(memory.block_weight_bytes(L70, 2) / bf16 - 0.25) < 0.02
+    assert abs(memory.block_weight_bytes(L70, 3) / bf16 - 0.25) < 0.02
 
 
 def test_decode_bytes_known_config():

@@ -177,3 +177,72 @@ def test_quantize_weight_dispatch(wq):
     ref = _exact(quant.bf16_to_f32(w))
     tol = {0: 0.0, 1: 0.02 / 127 * 4, 2: 0.02 / 15 * 8}[wq]
     assert np.max(np.abs(deq - ref)) <= tol
+
+
+# ---------------------------------------------------------------- GPTQ4 (act order)
+def _fixture_gptq4():
+    g = _golden("gptq4_act_order_example.json")
+    w = np.zeros((1, g["k"]), dtype=np.uint16)
+    for k, v in g["w_nonzero"].items():
+        w[0, int(k)] = v
+    perm = np.concatenate([np.arange(1, g["k"], 2), np.arange(0, g["k"], 2)]).astype(np.int32)
+    return g, w, perm
+
+
+def test_gptq4_hand_example():
+    """The act-order groups, their scale / zero, the act-order packing and the
+    channel-order dequantisation of the hand-worked fixture."""
+    g, w, perm = _fixture_gptq4()
+    p, s, z = quant.quantize_gptq4(w, perm)
+    assert s[0].tolist() == g["scale_bits"] and z[0].tolist() == g["zero_bits"]
+    for i, b in g["bytes_at"].items():
+        assert int(p[0, int(i)]) == b, i
+    d = quant.dequant_gptq4(p, s, z, perm)
+    for i, v in g["dequant_at"].items():
+        assert d[0, int(i)] == v, i
+    gi = quant.g_idx_of(perm)
+    assert np.all(gi[1::2] == 0) and np.all(gi[0::2] == 1)
+
+
+def test_gptq4_identity_order_is_int4():
+    """With the identity act order GPTQ4 is the int4 group-128 format, bit for bit."""
+    w = _weights(12, 512)
+    ident = np.arange(512, dtype=np.int32)
+    for a, b in zip(quant.quantize_gptq4(w, ident), quant.quantize_int4_g128(w)):
+        assert np.array_equal(a, b)
+    assert np.array_equal(quant.dequant_gptq4(*quant.quantize_gptq4(w, ident), ident),
+                          quant.dequant_int4(*quant.quantize_int4_g128(w)))
+
+
+def test_gptq4_groups_follow_the_act_order():
+    """Every group holds 128 channels, g_idx[perm[j]] = j // 128, and each
+    channel's error is at most half its own group's scale."""
+    k = 768
+    perm = synth.act_order(5, 1, 2, k)
+    gi = quant.g_idx_of(perm)
+    assert np.array_equal(np.bincount(gi), np.full(k // 128, 128))
+    assert np.array_equal(gi[perm], np.arange(k) // 128)
+    w = _weights(9, k)
+    p, s, z = quant.quantize_gptq4(w, perm)
+    err = np.abs(quant.dequant_gptq4(p, s, z, perm) - _exact(quant.bf16_to_f32(w)))
+    half = _exact(quant.bf16_to_f32(s))[:, gi] / 2
+    assert np.all(err <= half * (1 + 2 ** -20) + 1e-30)
+    q = quant.codes_gptq4(p, perm)
+    assert q.min() >= 0 and q.max() <= 15
+
+
+def test_gptq4_product_equals_reordered_int4_product():
+    """x W^T with W dequantised in channel order equals x[:, perm] W_a^T, W_a
+    the act-order storage read as plain int4: the identity the device uses.
+    A perm / inverse mix-up or a group taken in channel order fails it."""
+    k = 512
+    perm = synth.act_order(3, 0, 1, k)
+    assert not np.array_equal(perm[perm], np.arange(k))  # not an involution
+    w = _weights(6, k)
+    p, s, z = quant.quantize_gptq4(w, perm)
+    x = quant.bf16_to_f32(synth.uniform_bf16(4, 9, (5, k), -1.0, 1.0)).astype(np.float64)
+    y = x @ quant.dequant_gptq4(p, s, z, perm).T
+    ya = x[:, perm] @ quant.dequant_int4(p, s, z).T
+    assert np.allclose(y, ya, rtol=0, atol=1e-12)
+    # taking the groups in channel order instead gives different weights
+    assert not np.allclose(quant.dequant_gptq4(p, s, z, perm), quant.dequant_int4(p, s, z))

@@ -52,3 +52,27 @@ def test_bf16_rounding_nearest_even():
     # 1 + 2^-8 is a tie between 1 and 1 + 2^-7: to the even mantissa (1.0);
     # 1 + 3 * 2^-8 ties between 1 + 2^-7 and 1 + 2^-6: to 1 + 2^-6 (even)
     assert [hex(int(b)) for b in got] == ["0x3f80", "0x3f80", "0x3f82", "0x3f81", "0xc020", "0x4780"]
+
+
+def test_act_order_is_a_seeded_permutation():
+    """Fisher-Yates over counter-based draws: a permutation, a function of
+    (seed, layer, matrix) alone, and uniform over the 6 orders of 3 items."""
+    p = synth.act_order(0, 1, 2, 1000)
+    assert p.dtype == np.int32 and sorted(p.tolist()) == list(range(1000))
+    assert np.array_equal(p, synth.act_order(0, 1, 2, 1000))
+    assert not np.array_equal(p, synth.act_order(0, 1, 3, 1000))
+    assert not np.array_equal(p, synth.act_order(1, 1, 2, 1000))
+    counts = {}
+    for seed in range(3000):
+        t = tuple(synth.act_order(seed, 0, 0, 3).tolist())
+        counts[t] = counts.get(t, 0) + 1
+    assert len(counts) == 6
+    chi2 = sum((c - 500.0) ** 2 / 500.0 for c in counts.values())
+    assert chi2 < 25  # 5 degrees of freedom
+
+
+def test_act_order_first_swaps_by_hand():
+    """K = 2: one swap, j = multiply-shift of draw 0's high 32 bits onto [0, 1]."""
+    hi = int(synth.draws(7, synth.perm_stream(0, 0), 0, 1)[0]) >> 32
+    want = [1, 0] if (hi * 2) >> 32 == 0 else [0, 1]
+    assert synth.act_order(7, 0, 0, 2).tolist() == want
