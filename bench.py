@@ -48,8 +48,10 @@ CONFIGS = {
     "l7b": ((2, 4096, 32, 32, 128, 11008, 32000), 1, 0, 8, 512, 100),
     "l13b": ((2, 5120, 40, 40, 128, 13824, 32000), 2, 0, 16, 1024, 100),
     "l70b": ((2, 8192, 64, 8, 128, 28672, 32000), 2, 1, 32, 2048, 100),
+    # the 70B-shaped workload with GPTQ-format int4 weights (act-order groups)
+    "l70b_gptq4": ((2, 8192, 64, 8, 128, 28672, 32000), 3, 1, 32, 2048, 100),
 }
-WQ_NAME = {0: "bf16", 1: "int8-per-channel", 2: "int4-g128"}
+WQ_NAME = {0: "bf16", 1: "int8-per-channel", 2: "int4-g128", 3: "gptq4-g128-act-order"}
 KV_NAME = {0: "bf16", 1: "int8-per-token-head"}
 
 
@@ -62,7 +64,9 @@ def arch_dict(t):
 
 # ---------------------------------------------------------------- byte model
 def mat_bytes(n, k, wq):
-    return {0: 2 * n * k, 1: n * k + 2 * n, 2: n * k // 2 + 4 * n * (k // 128)}[wq]
+    """Stored bytes of one [n, k] matrix (GPTQ4: int4 plus the int32 act order)."""
+    return {0: 2 * n * k, 1: n * k + 2 * n, 2: n * k // 2 + 4 * n * (k // 128),
+            3: n * k // 2 + 4 * n * (k // 128) + 4 * k}[wq]
 
 
 def kernel_bytes(a, wq, kvq, B, ctx):
@@ -221,7 +225,7 @@ class ClockSampler:
 # decode.  The full shapes and the full batch are kept; where the workload's
 # prompt would make the untimed prefill set-up take minutes on the host
 # (the 70B-shaped prompt is 229 TFLOP at batch 32), a short prompt stands in.
-ORACLE_SAMPLE = {"tiny": (1, 32), "l7b": (8, 512), "l13b": (16, 64), "l70b": (32, 16)}
+ORACLE_SAMPLE = {"tiny": (1, 32), "l7b": (8, 512), "l13b": (16, 64), "l70b": (32, 16), "l70b_gptq4": (32, 16)}
 
 
 def oracle_sample(cfg, batch, prompt, steps, decode_tokens, warmup=0):
@@ -240,7 +244,8 @@ def oracle_sample(cfg, batch, prompt, steps, decode_tokens, warmup=0):
     get = lambda l, k, shape: (synth.f32_to_bf16_bits(np.ones(shape, np.float32)) if len(shape) == 1
                                else synth.weight_bf16(0, l, k, shape))
     with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as pool:  # set-up: quantise in parallel
-        w, _ = M.build_weights(arch, wq, get, map_fn=pool.map)
+        w, _ = M.build_weights(arch, wq, get, map_fn=pool.map,
+                               act_order=lambda l, m, k: synth.act_order(0, l, m, k))
     ref = M.Fingerprint(arch, w, kvq, batch, prompt + (warmup + steps) * decode_tokens + 1)
     toks = synth.tokens(0, batch * prompt, arch.vocab).reshape(batch, prompt)
     out = ref.prefill(toks)
@@ -365,7 +370,7 @@ def run_estimate(args, cfg):
 
     torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
     arch, wq, kvq, B, S, N = cfg
-    full = {"l7b": 32, "l13b": 40, "l70b": 80, "tiny": 4}[args.config]
+    full = {"l7b": 32, "l13b": 40, "l70b": 80, "l70b_gptq4": 80, "tiny": 4}[args.config]
     lens = (16, 64)
 
     def measure(L, n, iters):

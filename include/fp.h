@@ -51,8 +51,19 @@ extern "C" {
  *                     (bits 4i..4i+3) = element (0,2,4,6,1,3,5,7)[i], so the
  *                     nibbles a 0x000F000F mask picks are a consecutive pair;
  *                     + bf16 scale and bf16 zero per row and 128-wide group
- *                     of K, [N][K/128] each; w = (q - z) * s               */
-enum { FP_W_BF16 = 0, FP_W_INT8 = 1, FP_W_INT4_G128 = 2 };
+ *                     of K, [N][K/128] each; w = (q - z) * s
+ *   FP_W_GPTQ4      : GPTQ-format int4 with act order ("GPTQ4" in the same
+ *                     table): an act order perm, int32 [K], a permutation of
+ *                     the input channels; group g holds the channels
+ *                     perm[128g .. 128g+127] (GPTQ's g_idx[perm[j]] = j/128).
+ *                     Codes, scales and zeros are the FP_W_INT4_G128 layout
+ *                     of the matrix read in act order (stored column j is
+ *                     channel perm[j]): w[n][perm[j]] = (q[n][j] - z[n][j/128])
+ *                     * s[n][j/128].  Without calibration data the codes are
+ *                     the int4 rule on each group's values (round to nearest).
+ *                     fp_create draws one act order per fused matrix from the
+ *                     seed (Fisher-Yates over SplitMix64).                  */
+enum { FP_W_BF16 = 0, FP_W_INT8 = 1, FP_W_INT4_G128 = 2, FP_W_GPTQ4 = 3 };
 
 /* KV cache format (INT8 KV cache: table "Models and configurations").
  *   FP_KV_BF16 : K and V as bf16
@@ -104,7 +115,7 @@ typedef struct fp_handle fp_handle;
  *   stream      : cudaStream_t; NULL = a stream the handle creates and owns
  * Shape limits (FP_ERR_UNSUPPORTED): head_dim not 64/128; hidden not a
  * multiple of 64 or ffn not a multiple of 32 (both multiples of 128 with int4
- * weights); page_size != 16; n_layers > FP_MAX_LAYERS.
+ * or GPTQ4 weights); page_size != 16; n_layers > FP_MAX_LAYERS.
  * All device memory (weights, KV pages, activations for a prefill of
  * batch * max_context tokens, workspaces) is reserved here once; that sum is
  * the peak footprint fp_profile reports. */
@@ -234,7 +245,8 @@ enum {
   FP_G_LOGITS = 8,   /* fp32 [batch][vocab] of the last call                     */
   FP_G_TOKENS = 9,   /* int32 [batch] last emitted tokens                        */
   FP_G_PAGE_TABLE = 10, /* int32 [batch][pages_per_seq]                          */
-  FP_G_LENGTH = 11   /* int32 [batch] cached positions per sequence              */
+  FP_G_LENGTH = 11,  /* int32 [batch] cached positions per sequence              */
+  FP_G_W_PERM = 12   /* (layer, mat) int32 [K] act order of a GPTQ4 matrix         */
 };
 long long fp_get_tensor(fp_handle* h, int what, int layer, int mat, void* host_dst, size_t bytes);
 

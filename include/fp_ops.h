@@ -38,6 +38,15 @@ extern "C" {
 int fp_op_quantize(int wquant, const uint16_t* w, int N, int K, void* codes, uint16_t* scales,
                    uint16_t* zeros, void* stream);
 
+/* Quantise w [N][K] (bf16) into the FP_W_GPTQ4 format of fp.h: int4 over
+ * the act-order groups of perm (int32 [K], a permutation of 0..K-1; group g
+ * holds the channels perm[128g .. 128g+127]), codes stored in act order
+ * ([N][K/2], the int4 packing), scales and zeros bf16 [N][K/128]
+ * (GPTQ4, Sec. 3.2 and the table "Models and configurations").  K % 128 ==
+ * 0.  An entry of perm outside [0, K) reads as a zero weight. */
+int fp_op_quantize_gptq4(const uint16_t* w, int N, int K, const int32_t* perm, void* codes, uint16_t* scales,
+                         uint16_t* zeros, void* stream);
+
 /* Fill w [n] with the seeded bf16 weights of stream `stream_id` (SplitMix64
  * counter-based draws, Irwin-Hall(4), sigma 0.02; elements start..start+n-1). */
 int fp_op_init_weights(uint16_t* w, long long n, unsigned long long seed, long long stream_id,
@@ -79,6 +88,22 @@ int fp_op_linear(int wquant, int epilogue, const uint16_t* x, int M, int N, int 
                  const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
                  void* workspace, size_t workspace_bytes, void* stream);
 size_t fp_op_linear_workspace_bytes(int wquant, int M, int N, int K);
+
+/* The weight-only linear of fp_op_linear for FP_W_GPTQ4 weights (codes,
+ * scales, zeros as fp_op_quantize_gptq4 writes them; perm the act order).
+ * y = x W^T with W in channel order.  M <= 64: x is gathered into the act
+ * order in the workspace (one kernel) and the int4 decode linear runs on it;
+ * M > 64: the weights are expanded back into channel order (the inverse act
+ * order is computed into the workspace) and the prefill GEMM multiplies x as
+ * it is.  workspace: 256-byte aligned, at least
+ * fp_op_linear_gptq4_workspace_bytes(M, N, K) bytes, its leading ticket
+ * counters zero before the first call (every call leaves them zero).  An
+ * entry of perm outside [0, K) reads as zero and sets *err = 1 (err may be
+ * NULL).  K % 128 == 0 (FP_ERR_UNSUPPORTED). */
+int fp_op_linear_gptq4(int epilogue, const uint16_t* x, int M, int N, int K, const int32_t* perm, const void* codes,
+                       const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                       void* workspace, size_t workspace_bytes, int32_t* err, void* stream);
+size_t fp_op_linear_gptq4_workspace_bytes(int M, int N, int K);
 
 /* RMSNorm of selected rows: y[r] = x[r*row_stride + row_offset] /
  * sqrt(mean(x^2) + eps) * g, r < M; x, y, g bf16; fp32 arithmetic. */

@@ -138,7 +138,7 @@ def tensor_shape(arch: Arch, layer: int, tensor: int):
             (d,), (f, d), (f, d), (d, f)][tensor]
 
 
-def build_weights(arch: Arch, wquant: int, get_bf16, map_fn=map):
+def build_weights(arch: Arch, wquant: int, get_bf16, map_fn=map, act_order=None):
     """Quantise bf16 weights the way the configuration says.
 
     get_bf16(layer, tensor, shape) -> bf16 bit patterns.  Linear layers of
@@ -148,6 +148,8 @@ def build_weights(arch: Arch, wquant: int, get_bf16, map_fn=map):
     bf16.  Returns (fp64 weights for the forward pass, quantised payloads).
     ``map_fn`` applies the quantiser to the matrices (a thread pool's map
     spreads the large ones over cores; the result does not depend on it).
+    GPTQ4 (wquant 3) takes each fused matrix's act order from
+    ``act_order(layer, matrix, K)``, matrix 0..3 = Wqkv, Wo, Wgu, Wdown.
     """
     w, payload = {}, {}
     f64 = lambda b: quant.bf16_to_f32(b).astype(np.float64)
@@ -162,8 +164,9 @@ def build_weights(arch: Arch, wquant: int, get_bf16, map_fn=map):
                 "wo": raw["wo"],
                 "wgu": np.concatenate([raw["wgate"], raw["wup"]]),
                 "wdown": raw["wdown"]}
-        jobs += [((l, name), bits) for name, bits in mats.items()]
-    for (key, _), res in zip(jobs, map_fn(lambda j: quant.quantize_weight(j[1], wquant), jobs)):
+        jobs += [((l, name), bits, act_order(l, m, bits.shape[1]) if wquant == 3 else None)
+                 for m, (name, bits) in enumerate(mats.items())]
+    for (key, _, _), res in zip(jobs, map_fn(lambda j: quant.quantize_weight(j[1], wquant, j[2]), jobs)):
         payload[key], w[key] = res
     return w, payload
 

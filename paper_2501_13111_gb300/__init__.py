@@ -28,7 +28,7 @@ _lib = C.CDLL(LIB_PATH)
 # ------------------------------------------------------------------ constants
 FP_OK, FP_ERR_INVALID_ARG, FP_ERR_UNSUPPORTED, FP_ERR_OOM = 0, -1, -2, -3
 FP_ERR_CUDA, FP_ERR_CAPACITY, FP_ERR_DEVICE_ASSERT, FP_ERR_STATE = -4, -5, -6, -7
-FP_W_BF16, FP_W_INT8, FP_W_INT4_G128 = 0, 1, 2
+FP_W_BF16, FP_W_INT8, FP_W_INT4_G128, FP_W_GPTQ4 = 0, 1, 2, 3
 FP_KV_BF16, FP_KV_INT8 = 0, 1
 FP_FLAG_KEEP_HIDDEN, FP_FLAG_NO_INIT = 1, 2
 FP_MAX_LAYERS = 80
@@ -37,7 +37,7 @@ FP_MAX_LAYERS = 80
 FP_T_EMBED, FP_T_FINAL_NORM, FP_T_LM_HEAD = 0, 1, 2
 FP_M_QKV, FP_M_O, FP_M_GU, FP_M_DOWN = 0, 1, 2, 3
 (FP_G_W_CODES, FP_G_W_SCALES, FP_G_W_ZEROS, FP_G_K_POOL, FP_G_V_POOL, FP_G_K_SCALES, FP_G_V_SCALES,
- FP_G_HIDDEN, FP_G_LOGITS, FP_G_TOKENS, FP_G_PAGE_TABLE, FP_G_LENGTH) = range(12)
+ FP_G_HIDDEN, FP_G_LOGITS, FP_G_TOKENS, FP_G_PAGE_TABLE, FP_G_LENGTH, FP_G_W_PERM) = range(13)
 KERNEL_CLASSES = ("embed", "rmsnorm", "lin_qkv", "rope_kv", "attn", "attn_combine", "lin_o", "lin_gu",
                   "lin_down", "lm_head", "argmax")
 FP_K_COUNT = len(KERNEL_CLASSES)
@@ -136,6 +136,9 @@ _PROTOS = {
     "fp_op_init_weights": (_I, [_P, _LL, _ULL, _LL, _LL, _P]),
     "fp_op_linear": (_I, [_I, _I, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _SZ, _P]),
     "fp_op_linear_workspace_bytes": (_SZ, [_I, _I, _I, _I]),
+    "fp_op_quantize_gptq4": (_I, [_P, _I, _I, _P, _P, _P, _P, _P]),
+    "fp_op_linear_gptq4": (_I, [_I, _P, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _SZ, _P, _P]),
+    "fp_op_linear_gptq4_workspace_bytes": (_SZ, [_I, _I, _I]),
     "fp_op_rmsnorm": (_I, [_P, _I, _I, _I, _I, _P, _F, _P, _P]),
     "fp_op_embed": (_I, [_P, _I, _P, _I, _I, _P, _P, _P]),
     "fp_op_rope_table": (_I, [_I, _I, _F, _P, _P]),
@@ -286,6 +289,20 @@ def fp_op_init_weights(w, n, seed, stream_id, start=0, stream=None):
 
 def fp_op_linear_workspace_bytes(wquant, M, N, K):
     return _lib.fp_op_linear_workspace_bytes(wquant, M, N, K)
+
+
+def fp_op_quantize_gptq4(w, N, K, perm, codes, scales, zeros, stream=None):
+    return _check(_lib.fp_op_quantize_gptq4(w, N, K, perm, codes, scales, zeros, stream))
+
+
+def fp_op_linear_gptq4_workspace_bytes(M, N, K):
+    return _lib.fp_op_linear_gptq4_workspace_bytes(M, N, K)
+
+
+def fp_op_linear_gptq4(epilogue, x, M, N, K, perm, codes, scales, zeros, residual, y, workspace, workspace_bytes,
+                       err=None, stream=None):
+    return _check(_lib.fp_op_linear_gptq4(epilogue, x, M, N, K, perm, codes, scales, zeros, residual, y, workspace,
+                                          workspace_bytes, err, stream))
 
 
 def fp_op_linear(wquant, epilogue, x, M, N, K, codes, scales, zeros, residual, y, workspace=None,

@@ -260,8 +260,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // ------------------------------------------------------------------ dequant to bf16
 // int8: w = q (exact; the row scale is applied by the GEMM epilogue).
 // int4: w = bf16((q - z) * s), 8 elements (one packed word) per thread.
+// GPTQ4: the same expansion back into channel order: output channel k is
+// act-order column j = inv[k] (inv the inverse of the act order), with the
+// scale and zero of group j / 128; 8 consecutive channels per thread.
 __global__ void dequant_kernel(int wquant, const void* __restrict__ codes, const uint16_t* __restrict__ scales,
-                               const uint16_t* __restrict__ zeros, int N, int K, uint16_t* __restrict__ out) {
+                               const uint16_t* __restrict__ zeros, int N, int K, uint16_t* __restrict__ out,
+                               const int32_t* __restrict__ inv) {
   pdl_trigger();
   pdl_wait();
   const long long words = (long long)N * K / 8;
@@ -270,7 +274,17 @@ __global__ void dequant_kernel(int wquant, const void* __restrict__ codes, const
     const long long row = e0 / K;
     const int k0 = (int)(e0 % K);
     float f[8];
-    if (wquant == FP_W_INT8) {
+    if (wquant == FP_W_GPTQ4) {
+      const uint32_t* cw = (const uint32_t*)codes + row * (K / 8);
+      const long long g0 = row * (K / 128);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int a = min(max(inv[k0 + j], 0), K - 1);  // the inverse comes from the act order, in range
+        const int e = a & 7, nib = (e >> 1) + 4 * (e & 1);  // element e of a word sits in this nibble
+        const float q = (float)((cw[a >> 3] >> (4 * nib)) & 0xF);
+        f[j] = (q - bf2f(zeros[g0 + (a >> 7)])) * bf2f(scales[g0 + (a >> 7)]);
+      }
+    } else if (wquant == FP_W_INT8) {
       const uint2 c = *reinterpret_cast<const uint2*>((const int8_t*)codes + e0);
       const uint32_t w[2] = {c.x, c.y};
 #pragma unroll
@@ -400,18 +414,19 @@ static cudaError_t launch_tc_any(int epi, bool sc, const CUtensorMap& mx, const 
 
 // Expand rows [r0, r0 + rows) of a quantised matrix into out [rows][K] bf16.
 static cudaError_t dequant_rows(int wquant, const void* codes, const uint16_t* scales, const uint16_t* zeros, long long r0,
-                                int rows, int K, uint16_t* out, cudaStream_t s) {
+                                int rows, int K, uint16_t* out, const int32_t* inv, cudaStream_t s) {
+  const bool grouped = wquant == FP_W_INT4_G128 || wquant == FP_W_GPTQ4;
   const uint8_t* c = (const uint8_t*)codes + (wquant == FP_W_INT8 ? r0 * K : r0 * (K / 2));
-  const uint16_t* sc = wquant == FP_W_INT4_G128 ? scales + r0 * (K / 128) : scales;
-  const uint16_t* ze = wquant == FP_W_INT4_G128 ? zeros + r0 * (K / 128) : zeros;
+  const uint16_t* sc = grouped ? scales + r0 * (K / 128) : scales;
+  const uint16_t* ze = grouped ? zeros + r0 * (K / 128) : zeros;
   const long long words = (long long)rows * K / 8;
   const int blocks = (int)std::min<long long>((words + 255) / 256, 152 * 16);
-  return launch(dequant_kernel, dim3(blocks), dim3(256), 0, s, wquant, (const void*)c, sc, ze, rows, K, out);
+  return launch(dequant_kernel, dim3(blocks), dim3(256), 0, s, wquant, (const void*)c, sc, ze, rows, K, out, inv);
 }
 
 cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                            const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
-                           void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s) {
+                           void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s, const int32_t* inv) {
   const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
   const int Nout = nr == 2 ? N / 2 : N;
   const int wbox = epi == FP_EPI_SWIGLU ? 128 : 256;
@@ -429,8 +444,9 @@ cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N,
   const int band = band_cols(epi, N, K);
   for (int c0 = 0; c0 < Nout; c0 += band) {
     const int cols = std::min(band, Nout - c0);
-    FP_CUDA_TRY(dequant_rows(wquant, codes, scales, zeros, c0, cols, K, w, s));
-    if (nr == 2) FP_CUDA_TRY(dequant_rows(wquant, codes, scales, zeros, (long long)Nout + c0, cols, K, w + (size_t)cols * K, s));
+    FP_CUDA_TRY(dequant_rows(wquant, codes, scales, zeros, c0, cols, K, w, inv, s));
+    if (nr == 2)
+      FP_CUDA_TRY(dequant_rows(wquant, codes, scales, zeros, (long long)Nout + c0, cols, K, w + (size_t)cols * K, inv, s));
     if (!make_map(&mw, w, (long long)nr * cols, K, wbox)) return cudaErrorInvalidValue;
     const uint16_t* r = residual ? residual + c0 : nullptr;
     void* yb = epi == FP_EPI_F32 ? (void*)((float*)y + c0) : (void*)((uint16_t*)y + c0);

@@ -850,3 +850,58 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
 }
 
 }  // namespace fpk
+
+namespace fpk {
+
+// ---- GPTQ4 (int4 over an act order)
+// Decode (M <= 64): the workspace holds the int4 linear's own workspace
+// (ticket area first, kept at offset 0 whatever the shape) and then x in act
+// order, xp[m][j] = x[m][perm[j]]; the stored matrix is a plain int4 g128
+// matrix of the act-order channels, so y = xp W_stored^T.  Prefill: the
+// bf16 expansion puts each weight back in channel order (inv, the inverse
+// act order; computed into the workspace when the caller passes none) and
+// the GEMM multiplies x as it is.
+static size_t align256(size_t b) { return (b + 255) / 256 * 256; }
+
+static size_t gptq4_xp_offset(int M, int N, int K) {
+  return align256(std::max(linear_ws_bytes(FP_W_INT4_G128, M, N, K), counter_bytes(0)));
+}
+
+size_t linear_gptq4_ws_bytes(int M, int N, int K, bool with_inv) {
+  if (M <= 0 || N <= 0 || K <= 0) return 0;
+  if (M > 64) return align256(std::max(linear_ws_bytes(FP_W_INT4_G128, M, N, K), counter_bytes(0))) +
+                     (with_inv ? align256((size_t)K * 4) : 0);
+  return gptq4_xp_offset(M, N, K) + align256((size_t)M * K * 2);
+}
+
+size_t linear_gptq4_ws_bytes_upto(int max_m, int N, int K, bool with_inv) {
+  size_t w = 0;
+  for (int m = 1; m <= std::min(max_m, 64); ++m) w = std::max(w, linear_gptq4_ws_bytes(m, N, K, with_inv));
+  if (max_m > 64) w = std::max(w, linear_gptq4_ws_bytes(max_m, N, K, with_inv));
+  return w;
+}
+
+cudaError_t launch_linear_gptq4(int epi, const uint16_t* x, int M, int N, int K, const int32_t* perm,
+                                const int32_t* inv, const void* codes, const uint16_t* scales,
+                                const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
+                                cudaStream_t s, int32_t* err) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  if (!ws || ws_bytes < linear_gptq4_ws_bytes(M, N, K, inv == nullptr)) return cudaErrorInvalidValue;
+  if (M > 64) {
+    if (!gemm_tc_ok(M, N, K)) return cudaErrorInvalidValue;
+    const size_t lin = align256(std::max(linear_ws_bytes(FP_W_INT4_G128, M, N, K), counter_bytes(0)));
+    if (!inv) {
+      int32_t* tmp = (int32_t*)((char*)ws + lin);
+      FP_CUDA_TRY(launch_invert_perm(perm, K, tmp, err, s));
+      inv = tmp;
+    }
+    return launch_gemm_tc(FP_W_GPTQ4, epi, x, M, N, K, codes, scales, zeros, residual, y,
+                          (char*)ws + counter_bytes(0), lin - counter_bytes(0), err, s, inv);
+  }
+  uint16_t* xp = (uint16_t*)((char*)ws + gptq4_xp_offset(M, N, K));
+  FP_CUDA_TRY(launch_gather_cols(x, M, K, perm, xp, err, s));
+  return launch_linear(FP_W_INT4_G128, epi, xp, M, N, K, codes, scales, zeros, residual, y, ws,
+                       gptq4_xp_offset(M, N, K), s, err);
+}
+
+}  // namespace fpk

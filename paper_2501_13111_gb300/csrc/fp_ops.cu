@@ -38,6 +38,33 @@ int fp_op_quantize(int wquant, const uint16_t* w, int N, int K, void* codes, uin
   return cuda_status(launch_quantize(wquant, w, N, K, codes, scales, zeros, (cudaStream_t)stream));
 }
 
+int fp_op_quantize_gptq4(const uint16_t* w, int N, int K, const int32_t* perm, void* codes, uint16_t* scales,
+                         uint16_t* zeros, void* stream) {
+  if (N < 0 || K <= 0 || !w || !perm || !codes || !scales || !zeros) return FP_ERR_INVALID_ARG;
+  if (K % 128 != 0) return FP_ERR_UNSUPPORTED;
+  return cuda_status(launch_quantize(FP_W_GPTQ4, w, N, K, codes, scales, zeros, (cudaStream_t)stream, perm));
+}
+
+size_t fp_op_linear_gptq4_workspace_bytes(int M, int N, int K) {
+  if (M <= 0 || N <= 0 || K <= 0 || K % 128 != 0) return 0;
+  return linear_gptq4_ws_bytes(M, N, K, true);
+}
+
+int fp_op_linear_gptq4(int epilogue, const uint16_t* x, int M, int N, int K, const int32_t* perm, const void* codes,
+                       const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
+                       void* workspace, size_t workspace_bytes, int32_t* err, void* stream) {
+  if (M < 0 || N <= 0 || K <= 0 || !x || !perm || !codes || !scales || !zeros || !y) return FP_ERR_INVALID_ARG;
+  if (epilogue < FP_EPI_STORE || epilogue > FP_EPI_F32) return FP_ERR_INVALID_ARG;
+  if (epilogue == FP_EPI_RESID && !residual) return FP_ERR_INVALID_ARG;
+  if (epilogue == FP_EPI_SWIGLU && N % 2 != 0) return FP_ERR_INVALID_ARG;
+  if (K % 128 != 0) return FP_ERR_UNSUPPORTED;
+  if (M == 0) return FP_OK;
+  if (!workspace || workspace_bytes < linear_gptq4_ws_bytes(M, N, K, true) || ((uintptr_t)workspace & 255))
+    return FP_ERR_INVALID_ARG;
+  return cuda_status(launch_linear_gptq4(epilogue, x, M, N, K, perm, nullptr, codes, scales, zeros, residual, y,
+                                         workspace, workspace_bytes, (cudaStream_t)stream, err));
+}
+
 int fp_op_init_weights(uint16_t* w, long long n, unsigned long long seed, long long stream_id, long long start,
                        void* stream) {
   if (!w || n < 0 || start < 0) return FP_ERR_INVALID_ARG;

@@ -6,6 +6,8 @@
 // rounding decision uses IEEE fp32 division (__fdiv_rn) and rintf (ties to
 // even), so the codes are bit-identical to any other implementation of the
 // same definition.
+#include <algorithm>
+
 #include "common.cuh"
 #include "kernels.cuh"
 
@@ -71,18 +73,32 @@ __global__ void quantize_int8_kernel(const uint16_t* __restrict__ w, int K, int8
 // One warp per (row, 128-wide group); lane i holds elements 4i .. 4i+3.
 // mn = min(0, min w), mx = max(0, max w), s = bf16_ceil(fp32(fp32(mx - mn) / 15)),
 // z = clamp(rint(fp32(-mn / s)), 0, 15), q = clamp(rint(fp32(w / s)) + z, 0, 15).
+// perm (GPTQ4, may be NULL): element j of the stored row is input channel
+// perm[j], so group g holds channels perm[128 g .. 128 g + 127] (act order).
 __global__ void quantize_int4_kernel(const uint16_t* __restrict__ w, int N, int K, uint8_t* __restrict__ q,
-                                     uint16_t* __restrict__ scales, uint16_t* __restrict__ zeros) {
+                                     uint16_t* __restrict__ scales, uint16_t* __restrict__ zeros,
+                                     const int32_t* __restrict__ perm) {
   const int groups = K / 128;
   long long gid = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (gid >= (long long)N * groups) return;
   const int lane = threadIdx.x & 31;
   const long long row = gid / groups;
   const int g = (int)(gid % groups);
-  const uint16_t* wp = w + row * K + g * 128 + lane * 4;
-  uint2 raw = *reinterpret_cast<const uint2*>(wp);
-  float v[4] = {__uint_as_float(raw.x << 16), __uint_as_float(raw.x & 0xFFFF0000u),
-                __uint_as_float(raw.y << 16), __uint_as_float(raw.y & 0xFFFF0000u)};
+  float v[4];
+  if (perm) {
+    // an entry outside [0, K) reads as 0 (the act order must be a permutation)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int k = perm[g * 128 + lane * 4 + i];
+      v[i] = (unsigned)k < (unsigned)K ? bf2f(w[row * K + k]) : 0.f;
+    }
+  } else {
+    const uint2 raw = *reinterpret_cast<const uint2*>(w + row * K + g * 128 + lane * 4);
+    v[0] = __uint_as_float(raw.x << 16);
+    v[1] = __uint_as_float(raw.x & 0xFFFF0000u);
+    v[2] = __uint_as_float(raw.y << 16);
+    v[3] = __uint_as_float(raw.y & 0xFFFF0000u);
+  }
   float mn = fminf(fminf(v[0], v[1]), fminf(v[2], v[3]));
   float mx = fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3]));
 #pragma unroll
@@ -118,7 +134,7 @@ __global__ void quantize_int4_kernel(const uint16_t* __restrict__ w, int N, int 
 }
 
 cudaError_t launch_quantize(int wquant, const uint16_t* w, int N, int K, void* codes, uint16_t* scales,
-                            uint16_t* zeros, cudaStream_t s) {
+                            uint16_t* zeros, cudaStream_t s, const int32_t* perm) {
   if (N <= 0 || K <= 0) return cudaSuccess;
   if (wquant == FP_W_BF16) {
     return cudaMemcpyAsync(codes, w, (size_t)N * K * 2, cudaMemcpyDeviceToDevice, s);
@@ -128,7 +144,61 @@ cudaError_t launch_quantize(int wquant, const uint16_t* w, int N, int K, void* c
   }
   long long warps = (long long)N * (K / 128);
   int blocks = (int)((warps + 7) / 8);
-  return launch(quantize_int4_kernel, dim3(blocks), dim3(256), 0, s, w, N, K, (uint8_t*)codes, scales, zeros);
+  return launch(quantize_int4_kernel, dim3(blocks), dim3(256), 0, s, w, N, K, (uint8_t*)codes, scales, zeros,
+                wquant == FP_W_GPTQ4 ? perm : nullptr);
+}
+
+// ------------------------------------------------------------------ act order
+// xp[m][j] = x[m][perm[j]]: the activations in a GPTQ4 matrix's act order,
+// eight columns (one 16-byte store) per thread.  An entry of perm outside
+// [0, K) reads as 0 and sets *err = 1.
+__global__ void gather_cols_kernel(const uint16_t* __restrict__ x, int M, int K, const int32_t* __restrict__ perm,
+                                   uint16_t* __restrict__ xp, int32_t* err) {
+  pdl_trigger();
+  pdl_wait();
+  const long long units = (long long)M * (K / 8);
+  bool bad = false;
+  for (long long u = (long long)blockIdx.x * blockDim.x + threadIdx.x; u < units;
+       u += (long long)gridDim.x * blockDim.x) {
+    const long long m = u / (K / 8);
+    const int j0 = (int)(u % (K / 8)) * 8;
+    const uint16_t* xr = x + m * K;
+    uint32_t v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int k = perm[j0 + i];
+      const bool in = (unsigned)k < (unsigned)K;
+      bad |= !in;
+      v[i] = in ? (uint32_t)xr[k] : 0u;
+    }
+    *reinterpret_cast<uint4*>(xp + m * K + j0) =
+        make_uint4(v[0] | (v[1] << 16), v[2] | (v[3] << 16), v[4] | (v[5] << 16), v[6] | (v[7] << 16));
+  }
+  if (bad && err) atomicExch(err, 1);
+}
+
+// inv[perm[j]] = j; entries of perm outside [0, K) are skipped and set *err = 1
+__global__ void invert_perm_kernel(const int32_t* __restrict__ perm, int K, int32_t* __restrict__ inv, int32_t* err) {
+  pdl_trigger();
+  pdl_wait();
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < K; j += gridDim.x * blockDim.x) {
+    const int k = perm[j];
+    if ((unsigned)k < (unsigned)K) inv[k] = j;
+    else if (err) atomicExch(err, 1);
+  }
+}
+
+cudaError_t launch_gather_cols(const uint16_t* x, int M, int K, const int32_t* perm, uint16_t* xp, int32_t* err,
+                               cudaStream_t s) {
+  if (M <= 0 || K <= 0) return cudaSuccess;
+  const long long units = (long long)M * (K / 8);
+  const int blocks = (int)std::min<long long>((units + 255) / 256, 152 * 8);
+  return launch(gather_cols_kernel, dim3(blocks), dim3(256), 0, s, x, M, K, perm, xp, err);
+}
+
+cudaError_t launch_invert_perm(const int32_t* perm, int K, int32_t* inv, int32_t* err, cudaStream_t s) {
+  if (K <= 0) return cudaSuccess;
+  return launch(invert_perm_kernel, dim3(std::min((K + 255) / 256, 152 * 4)), dim3(256), 0, s, perm, K, inv, err);
 }
 
 }  // namespace fpk

@@ -34,6 +34,8 @@ struct Mat {
   void* codes = nullptr;
   uint16_t* scales = nullptr;
   uint16_t* zeros = nullptr;
+  int32_t* perm = nullptr;  // GPTQ4: the act order [K] and its inverse
+  int32_t* inv = nullptr;
   int N = 0, K = 0;
 };
 
@@ -47,13 +49,31 @@ struct Layer {
   float* vscale = nullptr;
 };
 
+// GPTQ4 stores an int4 g128 matrix (of the act-order channels) plus its act order
+bool grouped(int wq) { return wq == FP_W_INT4_G128 || wq == FP_W_GPTQ4; }
 size_t codes_bytes(int wq, long long N, long long K) {
   return wq == FP_W_BF16 ? N * K * 2 : wq == FP_W_INT8 ? N * K : N * K / 2;
 }
 size_t scale_bytes(int wq, long long N, long long K) {
   return wq == FP_W_BF16 ? 0 : wq == FP_W_INT8 ? N * 2 : N * (K / 128) * 2;
 }
-size_t zero_bytes(int wq, long long N, long long K) { return wq == FP_W_INT4_G128 ? N * (K / 128) * 2 : 0; }
+size_t zero_bytes(int wq, long long N, long long K) { return grouped(wq) ? N * (K / 128) * 2 : 0; }
+size_t perm_bytes(int wq, long long K) { return wq == FP_W_GPTQ4 ? K * 4 : 0; }
+
+// The act order of fused matrix m of block l: Fisher-Yates (Durstenfeld) over
+// the identity, swapping entry i = K-1 .. 1 with the multiply-shift of draw
+// K-1-i of stream (l + 1) * 16 + 9 + m onto [0, i] -- the definition the
+// input generators of the tests implement too.
+void act_order(unsigned long long seed, int l, int m, int K, int32_t* p) {
+  for (int j = 0; j < K; ++j) p[j] = j;
+  const uint64_t key = stream_key(seed, (uint64_t)(l + 1) * 16 + 9 + m);
+  for (int t = 0; t + 1 < K; ++t) {
+    const int i = K - 1 - t;
+    const uint64_t hi = mix64(key + (uint64_t)(t + 1) * kGamma) >> 32;
+    const int j = (int)((hi * (uint64_t)(i + 1)) >> 32);
+    std::swap(p[i], p[j]);
+  }
+}
 
 // Kernel-boundary event recorder for the instrumented (eager) decode pass.
 struct Tracer {
@@ -203,6 +223,9 @@ void carve(fp_handle* h, char* base) {
       size_t sb = scale_bytes(h->wq, M.N, M.K), zb = zero_bytes(h->wq, M.N, M.K);
       M.scales = sb ? c.take<uint16_t>(sb, &h->weight_bytes) : nullptr;
       M.zeros = zb ? c.take<uint16_t>(zb, &h->weight_bytes) : nullptr;
+      // the act order is part of the stored matrix; its inverse only serves the prefill expansion
+      M.perm = h->wq == FP_W_GPTQ4 ? c.take<int32_t>(perm_bytes(h->wq, M.K), &h->weight_bytes) : nullptr;
+      M.inv = h->wq == FP_W_GPTQ4 ? c.take<int32_t>(perm_bytes(h->wq, M.K), &h->ws_bytes) : nullptr;
     }
     L.kpool = c.take<void>(pool, &h->kv_bytes);
     L.vpool = c.take<void>(pool, &h->kv_bytes);
@@ -230,7 +253,9 @@ void carve(fp_handle* h, char* base) {
   h->attn_ws = c.take<void>(h->attn_ws_bytes, &h->ws_bytes);
   // every row count a forward can use: B (decode, LM head) and B * S for any prompt S
   size_t lw = 0;
-  for (int m = 0; m < 4; ++m) lw = std::max(lw, linear_ws_bytes_upto(h->wq, (int)R, NK[m][0], NK[m][1]));
+  for (int m = 0; m < 4; ++m)
+    lw = std::max(lw, h->wq == FP_W_GPTQ4 ? linear_gptq4_ws_bytes_upto((int)R, NK[m][0], NK[m][1], false)
+                                          : linear_ws_bytes_upto(h->wq, (int)R, NK[m][0], NK[m][1]));
   lw = std::max(lw, linear_ws_bytes_upto(FP_W_BF16, h->B, (int)V, (int)d));
   h->lin_ws_bytes = lw;
   h->lin_ws = lw ? c.take<void>(lw, &h->ws_bytes) : nullptr;
@@ -247,7 +272,7 @@ bool bad_shape(const fp_arch* a, int wq, std::string& why) {
     why = buf;
     return true;
   }
-  int hm = wq == FP_W_INT4_G128 ? 128 : 64, fm = wq == FP_W_INT4_G128 ? 128 : 32;
+  int hm = grouped(wq) ? 128 : 64, fm = grouped(wq) ? 128 : 32;
   if (a->hidden % hm || a->ffn % fm || (a->n_heads * a->head_dim) % hm) {
     snprintf(buf, sizeof buf, "hidden %d / ffn %d / heads*head_dim %d not multiples of %d / %d / %d",
              a->hidden, a->ffn, a->n_heads * a->head_dim, hm, fm, hm);
@@ -270,6 +295,18 @@ bool bad_shape(const fp_arch* a, int wq, std::string& why) {
     h->launches += 1;                                          \
     h->tr.after(cls);                                          \
   } while (0)
+
+// One block linear: the GPTQ4 path (its decode gather counts as a launch of
+// its own) or the weight-only linear of the handle's format.
+cudaError_t block_linear(fp_handle* h, int epi, const uint16_t* x, int M, const Mat& W, const uint16_t* R, void* y) {
+  if (h->wq == FP_W_GPTQ4) {
+    if (M <= 64) h->launches += 1;
+    return launch_linear_gptq4(epi, x, M, W.N, W.K, W.perm, W.inv, W.codes, W.scales, W.zeros, R, y, h->lin_ws,
+                               h->lin_ws_bytes, h->stream, h->err);
+  }
+  return launch_linear(h->wq, epi, x, M, W.N, W.K, W.codes, W.scales, W.zeros, R, y, h->lin_ws, h->lin_ws_bytes,
+                       h->stream, h->err);
+}
 
 // One forward pass over M = B * S rows (S tokens per sequence at positions
 // pos[b] .. pos[b] + S - 1); tok: device ids [M].  decode = (S == 1 and the
@@ -294,9 +331,7 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
     const fp_kv_view kv = h->kv(l);
     if (l > 0) LTRY(launch_rmsnorm(h->h, M, d, 1, 0, Ly.attn_norm, a.rms_eps, h->y, s), FP_K_RMSNORM);
     const Mat& Q = Ly.mat[FP_M_QKV];
-    LTRY(launch_linear(h->wq, FP_EPI_STORE, h->y, M, Q.N, Q.K, Q.codes, Q.scales, Q.zeros, nullptr, h->qkv,
-                       h->lin_ws, h->lin_ws_bytes, s, h->err),
-         FP_K_LIN_QKV);
+    LTRY(block_linear(h, FP_EPI_STORE, h->y, M, Q, nullptr, h->qkv), FP_K_LIN_QKV);
     LTRY(launch_rope_kv(h->qkv, B, S, h->n_qkv, a.n_heads, kv, h->pos, h->rope_cs, h->err, s), FP_K_ROPE_KV);
     if (decode) {
       cudaError_t e2 = cudaSuccess;
@@ -310,18 +345,12 @@ int forward(fp_handle* h, const int32_t* tok, int S, bool decode) {
       LTRY(launch_attention_prefill(h->qkv, h->n_qkv, B, S, a.n_heads, kv, h->att, h->err, s), FP_K_ATTN);
     }
     const Mat& O = Ly.mat[FP_M_O];
-    LTRY(launch_linear(h->wq, FP_EPI_RESID, h->att, M, O.N, O.K, O.codes, O.scales, O.zeros, h->h, h->h,
-                       h->lin_ws, h->lin_ws_bytes, s, h->err),
-         FP_K_LIN_O);
+    LTRY(block_linear(h, FP_EPI_RESID, h->att, M, O, h->h, h->h), FP_K_LIN_O);
     LTRY(launch_rmsnorm(h->h, M, d, 1, 0, Ly.ffn_norm, a.rms_eps, h->y, s), FP_K_RMSNORM);
     const Mat& GU = Ly.mat[FP_M_GU];
-    LTRY(launch_linear(h->wq, FP_EPI_SWIGLU, h->y, M, GU.N, GU.K, GU.codes, GU.scales, GU.zeros, nullptr, h->act,
-                       h->lin_ws, h->lin_ws_bytes, s, h->err),
-         FP_K_LIN_GU);
+    LTRY(block_linear(h, FP_EPI_SWIGLU, h->y, M, GU, nullptr, h->act), FP_K_LIN_GU);
     const Mat& D = Ly.mat[FP_M_DOWN];
-    LTRY(launch_linear(h->wq, FP_EPI_RESID, h->act, M, D.N, D.K, D.codes, D.scales, D.zeros, h->h, h->h,
-                       h->lin_ws, h->lin_ws_bytes, s, h->err),
-         FP_K_LIN_DOWN);
+    LTRY(block_linear(h, FP_EPI_RESID, h->act, M, D, h->h, h->h), FP_K_LIN_DOWN);
     if (h->hidden) {
       cudaError_t e = cudaMemcpyAsync(h->hidden + (size_t)l * h->max_rows * d, h->h, (size_t)M * d * 2,
                                       cudaMemcpyDeviceToDevice, s);
@@ -432,7 +461,7 @@ int init_weights(fp_handle* h, uint16_t* staging) {
         e = launch_init_weights(staging + r0 * M.K, rows[m][p] * M.K, h->seed, base + parts[m][p], 0, s);
         r0 += rows[m][p];
       }
-      if (e == cudaSuccess) e = launch_quantize(h->wq, staging, M.N, M.K, M.codes, M.scales, M.zeros, s);
+      if (e == cudaSuccess) e = launch_quantize(h->wq, staging, M.N, M.K, M.codes, M.scales, M.zeros, s, M.perm);
       // the staging buffer is reused by the next matrix: keep the order
       if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     }
@@ -479,7 +508,7 @@ int fp_create(const fp_arch* arch, int wquant, int kvquant, int batch, int max_c
       a.vocab <= 0 || !(a.rms_eps >= 0.f) || !(a.rope_base > 0.f))
     return create_fail(nullptr, FP_ERR_INVALID_ARG, "non-positive shape field or bad eps / rope base");
   if (a.n_heads % a.n_kv_heads != 0) return create_fail(nullptr, FP_ERR_INVALID_ARG, "n_heads % n_kv_heads != 0");
-  if (wquant < FP_W_BF16 || wquant > FP_W_INT4_G128) return create_fail(nullptr, FP_ERR_INVALID_ARG, "wquant");
+  if (wquant < FP_W_BF16 || wquant > FP_W_GPTQ4) return create_fail(nullptr, FP_ERR_INVALID_ARG, "wquant");
   if (kvquant != FP_KV_BF16 && kvquant != FP_KV_INT8) return create_fail(nullptr, FP_ERR_INVALID_ARG, "kvquant");
   if (batch < 1 || max_context < 1) return create_fail(nullptr, FP_ERR_INVALID_ARG, "batch and max_context >= 1");
   if (alloc && (!alloc->alloc || !alloc->free)) return create_fail(nullptr, FP_ERR_INVALID_ARG, "allocator fields");
@@ -547,6 +576,20 @@ int fp_create(const fp_arch* arch, int wquant, int kvquant, int batch, int max_c
   if (e != cudaSuccess) return create_fail(h, FP_ERR_CUDA, "page table upload");
   int st = fp_op_rope_table(h->pps * h->P, a.head_dim, a.rope_base, h->rope_cs, h->stream);
   if (st) return create_fail(h, st, "rope table");
+  if (wquant == FP_W_GPTQ4) {
+    // every matrix's act order, drawn from the seed on the host, and its inverse
+    std::vector<int32_t> perm;
+    for (int l = 0; l < a.n_layers && e == cudaSuccess; ++l)
+      for (int m = 0; m < 4 && e == cudaSuccess; ++m) {
+        const Mat& M = h->L[l].mat[m];
+        perm.resize((size_t)M.K);
+        act_order(seed, l, m, M.K, perm.data());
+        e = cudaMemcpyAsync(M.perm, perm.data(), (size_t)M.K * 4, cudaMemcpyHostToDevice, h->stream);
+        if (e == cudaSuccess) e = launch_invert_perm(M.perm, M.K, M.inv, nullptr, h->stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);  // the host buffer is reused
+      }
+    if (e != cudaSuccess) return create_fail(h, FP_ERR_CUDA, "act orders");
+  }
 
   if (!(flags & FP_FLAG_NO_INIT)) {
     size_t stage = 0;
@@ -635,7 +678,7 @@ int fp_set_weight(fp_handle* h, int layer, int tensor, const uint16_t* host_bf16
   uint16_t* sc = M.scales ? (uint16_t*)((char*)M.scales + scale_bytes(wq, r0, M.K)) : nullptr;
   uint16_t* zr = M.zeros ? (uint16_t*)((char*)M.zeros + zero_bytes(wq, r0, M.K)) : nullptr;
   e = cudaMemcpyAsync(staging, host_bf16, (size_t)rows * M.K * 2, cudaMemcpyHostToDevice, s);
-  if (e == cudaSuccess) e = launch_quantize(wq, staging, (int)rows, M.K, codes, sc, zr, s);
+  if (e == cudaSuccess) e = launch_quantize(wq, staging, (int)rows, M.K, codes, sc, zr, s, M.perm);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   h->dev_free(staging);
   return e == cudaSuccess ? FP_OK : h->cuda_fail(e, "set weight");
@@ -730,7 +773,7 @@ long long fp_get_tensor_at(fp_handle* h, int what, int layer, int mat, size_t of
   if (!h) return FP_ERR_INVALID_ARG;
   const void* src = nullptr;
   size_t n = 0;
-  const bool per_layer = what <= FP_G_HIDDEN;
+  const bool per_layer = what <= FP_G_HIDDEN || what == FP_G_W_PERM;
   if (per_layer && (layer < 0 || layer >= h->a.n_layers)) return h->fail(FP_ERR_INVALID_ARG, "layer out of range");
   const size_t pool = (size_t)h->n_pages * h->a.n_kv_heads * h->P * h->a.head_dim * (h->kvq == FP_KV_BF16 ? 2 : 1);
   const size_t spool = (size_t)h->n_pages * h->a.n_kv_heads * h->P * 4;
@@ -743,6 +786,13 @@ long long fp_get_tensor_at(fp_handle* h, int what, int layer, int mat, size_t of
       if (what == FP_G_W_CODES) { src = M.codes; n = codes_bytes(h->wq, M.N, M.K); }
       else if (what == FP_G_W_SCALES) { src = M.scales; n = scale_bytes(h->wq, M.N, M.K); }
       else { src = M.zeros; n = zero_bytes(h->wq, M.N, M.K); }
+      break;
+    }
+    case FP_G_W_PERM: {
+      if (mat < 0 || mat > 3) return h->fail(FP_ERR_INVALID_ARG, "mat out of range");
+      const Mat& M = h->L[layer].mat[mat];
+      src = M.perm;
+      n = perm_bytes(h->wq, M.K);
       break;
     }
     case FP_G_K_POOL: src = h->L[layer].kpool; n = pool; break;
@@ -776,7 +826,8 @@ static unsigned long long block_matrix_bytes(const fp_handle* h) {
   unsigned long long t = 0;
   for (int m = 0; m < 4; ++m) {
     const Mat& M = h->L[0].mat[m];
-    t += codes_bytes(h->wq, M.N, M.K) + scale_bytes(h->wq, M.N, M.K) + zero_bytes(h->wq, M.N, M.K);
+    t += codes_bytes(h->wq, M.N, M.K) + scale_bytes(h->wq, M.N, M.K) + zero_bytes(h->wq, M.N, M.K) +
+         perm_bytes(h->wq, M.K);
   }
   return t;
 }

@@ -14,8 +14,14 @@ namespace fpk {
 // ---- weights: seeded fill and quantisers (fp_quant.cu)
 cudaError_t launch_init_weights(uint16_t* w, long long n, unsigned long long seed, long long stream_id,
                                 long long start, cudaStream_t s);
+// perm: the act order of a GPTQ4 matrix (ignored for the other formats)
 cudaError_t launch_quantize(int wquant, const uint16_t* w, int N, int K, void* codes, uint16_t* scales,
-                            uint16_t* zeros, cudaStream_t s);
+                            uint16_t* zeros, cudaStream_t s, const int32_t* perm = nullptr);
+// xp[m][j] = x[m][perm[j]] (K % 8 == 0); inv[perm[j]] = j.  Entries of perm
+// outside [0, K) set *err = 1 (err may be NULL).
+cudaError_t launch_gather_cols(const uint16_t* x, int M, int K, const int32_t* perm, uint16_t* xp, int32_t* err,
+                               cudaStream_t s);
+cudaError_t launch_invert_perm(const int32_t* perm, int K, int32_t* inv, int32_t* err, cudaStream_t s);
 
 // ---- small row kernels (fp_rows.cu)
 cudaError_t launch_embed(const int32_t* tok, int M, const uint16_t* E, int V, int d, uint16_t* h,
@@ -57,6 +63,16 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
                           const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
                           void* ws, size_t ws_bytes, cudaStream_t s, int32_t* err = nullptr);
 
+// GPTQ4 linear (fp_linear.cu): decode gathers x into the act order, prefill
+// expands the weights back into channel order.  inv may be NULL (computed
+// into the workspace, which is then K * 4 bytes larger for M > 64).
+size_t linear_gptq4_ws_bytes(int M, int N, int K, bool with_inv);
+size_t linear_gptq4_ws_bytes_upto(int max_m, int N, int K, bool with_inv);
+cudaError_t launch_linear_gptq4(int epi, const uint16_t* x, int M, int N, int K, const int32_t* perm,
+                                const int32_t* inv, const void* codes, const uint16_t* scales,
+                                const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
+                                cudaStream_t s, int32_t* err);
+
 // ---- int4 decode linear at 9-64 tokens on tcgen05 (fp_gemv_tc.cu)
 bool q4tc_ok(int wquant, int epi, int M, int N, int K);
 size_t q4tc_ws_bytes(int epi, int M, int N, int K);
@@ -67,9 +83,10 @@ cudaError_t launch_q4tc(int epi, const uint16_t* x, int M, int N, int K, const v
 // ---- prefill GEMM on tcgen05 (fp_gemm_tc.cu)
 bool gemm_tc_ok(int M, int N, int K);
 size_t gemm_tc_ws_bytes(int wquant, int N, int K);
+// inv: the inverse act order of a GPTQ4 matrix (its expansion returns to channel order)
 cudaError_t launch_gemm_tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
                            const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y,
-                           void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s);
+                           void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s, const int32_t* inv = nullptr);
 
 // ---- prefill GEMM with int8 / int4 weights dequantised in the kernel (fp_gemm_wq.cu)
 bool gemm_wq_ok(int wquant, int epi, int M, int N, int K, const void* x, const void* codes);

@@ -87,6 +87,40 @@ def case_linear(wq, epi, M, N, K, scratch=True, *, single, iters):
     return ms, moved / ms / 1e6, "GB/s"
 
 
+def case_linear_gptq4(epi, M, N, K, *, single, iters):
+    """GPTQ4 linear (fp_op_linear_gptq4): decode gathers x into the act order
+    before the int4 linear; prefill expands the weights back into channel order."""
+    nbytes = weight_bytes(N, K, 2) + 4 * K
+    copies = 1 if single else max(2, min(8, -(-3 * L2_BYTES // nbytes)))
+    perm = torch.randperm(K, device="cuda").to(torch.int32)
+    mats = []
+    for _ in range(copies):
+        w = torch.randint(-3000, 3000, (N * K,), dtype=torch.int16, device="cuda")
+        w = (w.to(torch.float32) * 1e-5).to(torch.bfloat16).view(torch.int16)
+        codes = torch.empty(N * K // 2, dtype=torch.uint8, device="cuda")
+        sc = torch.zeros(N * (K // 128), dtype=torch.int16, device="cuda")
+        ze = torch.zeros(N * (K // 128), dtype=torch.int16, device="cuda")
+        fp.fp_op_quantize_gptq4(w.data_ptr(), N, K, perm.data_ptr(), codes.data_ptr(), sc.data_ptr(), ze.data_ptr())
+        mats.append((codes, sc, ze))
+    x = torch.randn(M, K, device="cuda").to(torch.bfloat16)
+    nout = N // 2 if epi == 2 else N
+    y = torch.zeros(M * nout * 4, dtype=torch.uint8, device="cuda")
+    r = torch.zeros(M * nout, dtype=torch.bfloat16, device="cuda")
+    wsb = fp.fp_op_linear_gptq4_workspace_bytes(M, N, K)
+    ws = torch.zeros(max(wsb, 256), dtype=torch.uint8, device="cuda")
+
+    def f():
+        for codes, sc, ze in mats:
+            fp.fp_op_linear_gptq4(epi, x.data_ptr(), M, N, K, perm.data_ptr(), codes.data_ptr(), sc.data_ptr(),
+                                  ze.data_ptr(), r.data_ptr(), y.data_ptr(), ws.data_ptr(), wsb)
+
+    ms = timed(f, iters) / copies
+    moved = nbytes + 2 * M * K + 2 * M * nout + (2 * M * nout if epi == 1 else 0)
+    if M > 64:
+        return ms, 2.0 * M * N * K / (ms * 1e-3) / 1e12, "TFLOP/s"
+    return ms, moved / ms / 1e6, "GB/s"
+
+
 def case_attention(B, H, Hkv, hd, ctx, kvq, single, iters):
     P = 16
     pps = -(-ctx // P)
@@ -191,13 +225,18 @@ CASES["70b-qkv-prefill"] = ("linear", (2, 0, 65536, 10240, 8192))
 CASES["70b-gu-prefill"] = ("linear", (2, 2, 65536, 57344, 8192))
 CASES["70b-down-prefill"] = ("linear", (2, 1, 65536, 8192, 28672))
 CASES["bf16-8k-prefill"] = ("linear", (0, 0, 8192, 8192, 8192))
+# the 70B-shaped block's linears with GPTQ4 weights, decode (M 32) and prefill
+for _tag, (_epi, _n, _k) in {"qkv": (0, 10240, 8192), "o": (1, 8192, 8192), "gu": (2, 57344, 8192),
+                             "down": (1, 8192, 28672)}.items():
+    CASES[f"70b-gptq4-{_tag}"] = ("linear_gptq4", (_epi, 32, _n, _k))
+CASES["70b-gptq4-gu-prefill"] = ("linear_gptq4", (2, 65536, 57344, 8192))
 # the same quantised prefill linears without a workspace: dequantised inside the GEMM
 for _name in ["7b-qkv-prefill", "7b-gu-prefill", "7b-down-prefill", "13b-gu-prefill", "70b-qkv-prefill",
               "70b-gu-prefill", "70b-down-prefill"]:
     CASES[_name + "-inkernel"] = ("linear", CASES[_name][1] + (False,))
 
-RUNNERS = {"linear": case_linear, "attention": case_attention, "attention_prefill": case_attention_prefill,
-           "argmax": case_argmax}
+RUNNERS = {"linear": case_linear, "linear_gptq4": case_linear_gptq4, "attention": case_attention,
+           "attention_prefill": case_attention_prefill, "argmax": case_argmax}
 
 
 def main(argv=None):

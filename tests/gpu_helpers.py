@@ -9,8 +9,8 @@ from oracle import model as M
 from oracle import quant
 
 # Tolerances of the parity bar: max |gpu - ref| <= tau * max |ref| per tensor,
-# 2e-2 on bf16 / int8 weight paths, 5e-2 on int4 weight paths.
-TAU = {0: 2e-2, 1: 2e-2, 2: 5e-2}
+# 2e-2 on bf16 / int8 weight paths, 5e-2 on int4 weight paths (GPTQ4 is int4).
+TAU = {0: 2e-2, 1: 2e-2, 2: 5e-2, 3: 5e-2}
 
 
 def torch_mod():

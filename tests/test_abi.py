@@ -53,6 +53,7 @@ def _arch(**kw):
     (dict(n_layers=81), 0, -2),
     (dict(hidden=520), 0, -2),
     (dict(ffn=1376), 2, -2),   # int4 needs ffn % 128
+    (dict(ffn=1376), 3, -2),   # so does GPTQ4
     (dict(n_heads=32, n_kv_heads=2), 0, -2),  # group of 16 is not built
     (dict(vocab=0), 0, -1),
 ])
@@ -63,7 +64,7 @@ def test_create_rejects_bad_shapes_on_host(fp, kw, wq, code):
 
 
 def test_create_rejects_bad_modes_on_host(fp):
-    for args in [(_arch(), 3, 0, 1, 64), (_arch(), 0, 2, 1, 64), (_arch(), 0, 0, 0, 64), (_arch(), 0, 0, 1, 0)]:
+    for args in [(_arch(), 4, 0, 1, 64), (_arch(), 0, 2, 1, 64), (_arch(), 0, 0, 0, 64), (_arch(), 0, 0, 1, 0)]:
         with pytest.raises(fp.FPError) as e:
             fp.fp_create(*args)
         assert e.value.code == fp.FP_ERR_INVALID_ARG
@@ -77,6 +78,12 @@ def test_op_argument_checks_on_host(fp):
     assert fp._lib.fp_op_linear(5, 0, 1, 1, 8, 8, 1, 1, 1, None, 1, None, 0, None) == -1
     # int4 needs K % 128
     assert fp._lib.fp_op_linear(2, 0, 1, 1, 8, 64, 1, 1, 1, None, 1, None, 0, None) == -2
+    # GPTQ4: the act order is required, K % 128, a workspace
+    assert fp._lib.fp_op_linear_gptq4(0, 1, 1, 8, 128, None, 1, 1, 1, None, 1, 1, 1 << 20, None, None) == -1
+    assert fp._lib.fp_op_linear_gptq4(0, 1, 1, 8, 64, 1, 1, 1, 1, None, 1, 1, 1 << 20, None, None) == -2
+    assert fp._lib.fp_op_linear_gptq4(0, 1, 1, 8, 128, 1, 1, 1, 1, None, 1, None, 0, None, None) == -1
+    assert fp._lib.fp_op_quantize_gptq4(1, 8, 128, None, 1, 1, 1, None) == -1
+    assert fp._lib.fp_op_quantize_gptq4(1, 8, 64, 1, 1, 1, 1, None) == -2
     assert fp._lib.fp_op_quantize(2, 1, 4, 100, 1, 1, 1, None) == -2
     assert fp._lib.fp_op_rmsnorm(1, 1, 12, 1, 0, 1, 1e-5, 1, None) == -2
     kv = fp.fp_kv_view(0, 2, 96, 16, 4, 8, 1, 1, None, None, 1)
