@@ -199,9 +199,13 @@ int fp_op_attention_decode_noalloc(const uint16_t* q, int q_stride, int B, int n
  * out bf16 [B*S][n_heads*head_dim].  head_dim 128 with 16-token pages,
  * 16-byte aligned q (q_stride a multiple of 8) and pools runs on tcgen05
  * (scores and output accumulated in TMEM); other shapes on mma.sync.  An
- * int8 cache enters as its codes (exact in bf16), with each key's K scale
- * multiplying its score column and its V scale its probability column in
- * fp32.  A page id outside [0, n_pages) reads zeros and sets *err = 1. */
+ * int8 cache enters as its codes, with each key's K scale multiplying its
+ * score column and its V scale its probability column in fp32; on tcgen05
+ * the int8-cache products run in fp16 (codes exact, q converted, P carrying
+ * the V scales times a power of two that keeps it in the fp16 normal
+ * range), and a q element beyond the fp16 range sets *err = 3 (the output
+ * is then invalid).  A page id outside [0, n_pages) reads zeros and sets
+ * *err = 1. */
 int fp_op_attention_prefill(const uint16_t* q, int q_stride, int B, int S, int n_heads,
                             const fp_kv_view* kv, uint16_t* out, int32_t* err, void* stream);
 

@@ -20,13 +20,20 @@
 //               already read.  The reference maximum m only moves when a tile
 //               raises it by more than 2^8 (O and the row sum are rescaled
 //               then); P never exceeds 256, and o / l is exact either way.
-//   int8 cache: warps 0, 6 and 7 (after warp 0 has issued the Q copy) widen
-//               the codes: each loads its rows' 16-byte code chunks, turns
-//               them into bf16 (integers of at most 8 bits: exact) in the
-//               same swizzled layout the TMA writes, and stages the tile's K
-//               and V scales; the softmax multiplies each score column by
-//               its K scale and each P column by its V scale (the row sum
-//               takes the unscaled P), so the scales enter in fp32.
+//   int8 cache: both products run on fp16 operands.  Warps 0, 6 and 7
+//               (after warp 0 has issued the Q copy) convert the Q tile to
+//               fp16 in place once, then widen the codes: each loads its
+//               rows' 16-byte code chunks and turns each pair into the fp16
+//               pair (1024 + q + 128) by one byte permute, minus 1152 --
+//               exact -- in the same swizzled layout the TMA writes, and
+//               stages the tile's K scales and its V scales times 2^sigma;
+//               the softmax multiplies each score column by its K scale and
+//               each P column by its scaled V scale in fp32 (the row sum
+//               takes the unscaled P) and packs P as fp16.  sigma, one per
+//               CTA, is the largest power of two keeping 256 * (largest V
+//               scale of the sequence) * 2^sigma within 65280, so P stays in
+//               the fp16 normal range; the output divides it out.  A q beyond
+//               the fp16 range sets status 3.
 // TMEM columns: scores S [0, 128) with P over [0, 64), O [128, 256).  Every
 // mbarrier wait is bounded (error 2 past the limit); a page id out of range
 // reads zeros and sets error 1.
@@ -87,10 +94,20 @@ FP_DEV uint32_t pa_pack(float lo, float hi) {
   return r;
 }
 
-// Signed byte `i` (0..3) of `w` as an exact fp32: 2^23 + (byte ^ 0x80) built
-// by a byte permute, then the offset subtracted.
-FP_DEV float pa_i8f(uint32_t w, int i) {
-  return __uint_as_float(__byte_perm(w ^ 0x80808080u, 0x4B000000u, 0x7650 | i)) - 8388736.f;
+// (lo, hi) -> fp16x2, round to nearest even.
+FP_DEV uint32_t pa_pack_h(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Signed bytes a and b of w as the fp16 pair (q_a, q_b), exact: the byte
+// permute places q + 128 under the fp16 exponent of 1024 (0x64nn = 1024 + nn),
+// one fp16x2 subtraction of 1152 leaves q.
+FP_DEV uint32_t pa_i8h2(uint32_t u, uint32_t sel) {
+  uint32_t h = __byte_perm(u, 0x64646464u, sel);
+  asm("sub.rn.f16x2 %0, %0, %1;" : "+r"(h) : "r"(0x64806480u));
+  return h;
 }
 
 template <bool KV8>
@@ -102,7 +119,9 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
                            const int32_t* __restrict__ page_table, int pages_per_seq, int n_pages,
                            uint16_t* __restrict__ out, int32_t* err) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t qfull, kfull, kempty, vfull, vempty, sfull, pfull, ofull, mma_done;
+  __shared__ uint64_t qfull, qconv, kfull, kempty, vfull, vempty, sfull, pfull, ofull, mma_done;
+  __shared__ float s_vmax[KV8 ? 3 : 1];  // int8: the widening warps' largest V scales
+  __shared__ float s_unscale;             // int8: 2^-sigma, removed from the output
   __shared__ uint32_t tmem_base;
   __shared__ int abort_word;
   __shared__ __align__(16) float s_scl[KV8 ? 4 * kPaB : 4];  // int8: [K, V][tile parity][key] scales
@@ -124,6 +143,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
   pdl_trigger();
   if (threadIdx.x == 0) {
     mbar_init(&qfull, 1);
+    mbar_init(&qconv, kPaWiden);  // int8: the widening warps converted Q to fp16
     mbar_init(&kfull, KV8 ? kPaWiden : 1);
     mbar_init(&kempty, 1);
     mbar_init(&vfull, KV8 ? kPaWiden : 1);
@@ -157,12 +177,50 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
     const int wi = (warp == 0 ? 0 : warp - 5) * 32 + lane;  // 0 .. 95
     const int c = wi & 7;                                     // code chunk: head_dim 16c .. 16c + 15
     const int rbase = wi >> 3;                                // tile rows rbase + 12i (< 128)
+    const int32_t* ptv = page_table + (long long)b * pages_per_seq;
+    // sigma: from the largest V scale over the keys this CTA reads
+    float vmax = 0.f;
+    const int nkeys = min(q0 + kPaB, S);
+    for (int key = wi; key < nkeys; key += 32 * kPaWiden) {
+      const int pg = __ldg(ptv + key / page_size);
+      if (pg >= 0 && pg < n_pages) vmax = fmaxf(vmax, __ldg(v_scale + (pg * Hkv + kvh) * page_size + key % page_size));
+    }
+    vmax = warp_max(vmax);
+    if (lane == 0) s_vmax[warp == 0 ? 0 : warp - 5] = vmax;
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * kPaWiden) : "memory");
+    vmax = fmaxf(fmaxf(s_vmax[0], s_vmax[1]), s_vmax[2]);
+    // 2^sigma with 256 * vmax * 2^sigma <= 65280 (vmax = 0: no V weight at all)
+    const int sigma = vmax > 0.f ? min(60, max(-60, (int)floorf(log2f(255.f / vmax)))) : 0;
+    const float vmul = exp2f((float)sigma);
+    // published before the first code tile, which every softmax wait follows
+    if (wi == 0) s_unscale = exp2f((float)-sigma);
+    // Q to fp16 in place (the element order of the swizzled tile is kept)
+    bool ok = __all_sync(0xffffffffu, mbar_wait(&qfull, 0));
+    if (ok) {
+      bool over = false;
+      for (int i = wi; i < kPaTile / 16; i += 32 * kPaWiden) {
+        uint4* p = reinterpret_cast<uint4*>(sQ) + i;
+        const uint4 v = *p;
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+        uint32_t o[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 f = bf2x2f(w4[j]);
+          over |= fabsf(f.x) > 65504.f || fabsf(f.y) > 65504.f;
+          o[j] = pa_pack_h(f.x, f.y);
+        }
+        *p = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+      if (over && err) atomicExch(err, 3);  // q outside the fp16 range: the output is invalid
+      fence_proxy_async();
+    }
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&qconv);
     // its bf16 form is chunks cb, cb + 1 of half c / 4 of the swizzled row;
     // the lanes of the upper half store the odd chunk first, so the eight
     // lanes of one row write eight distinct 16-byte bank groups
     const int cb = 2 * (c & 3), half_off = (c >> 2) * kPaHalf;
-    const int32_t* pt = page_table + (long long)b * pages_per_seq;
-    bool ok = true;
+    const int32_t* pt = ptv;
     for (int t = 0; t < nt && ok; ++t) {
       int rowi[kPaWRows];  // pool row of each of the thread's keys (< 2^31); -1 reads zeros
 #pragma unroll
@@ -181,7 +239,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
 #pragma unroll
       for (int i = 0; i < kPaWRows; ++i) {
         sck[i] = (c == 0 && rowi[i] >= 0) ? __ldg(k_scale + rowi[i]) : 0.f;
-        scv[i] = (c == 0 && rowi[i] >= 0) ? __ldg(v_scale + rowi[i]) : 0.f;
+        scv[i] = (c == 0 && rowi[i] >= 0) ? __ldg(v_scale + rowi[i]) * vmul : 0.f;
       }
 #pragma unroll 1
       for (int which = 0; which < 2; ++which) {
@@ -201,11 +259,11 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
         for (int i = 0; i < kPaWRows; ++i) {
           const int row = rbase + 4 * kPaWiden * i, sw = row & 7;
           if (row >= kPaB) break;
-          const uint32_t ww[4] = {w[i].x, w[i].y, w[i].z, w[i].w};
+          const uint32_t ww[4] = {w[i].x ^ 0x80808080u, w[i].y ^ 0x80808080u, w[i].z ^ 0x80808080u,
+                                  w[i].w ^ 0x80808080u};
           uint32_t o[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            o[j] = pa_pack(pa_i8f(ww[j >> 1], (2 * j) & 3), pa_i8f(ww[j >> 1], (2 * j + 1) & 3));
+          for (int j = 0; j < 8; ++j) o[j] = pa_i8h2(ww[j >> 1], (j & 1) ? 0x4342 : 0x4140);
           const uint4 e = make_uint4(o[0], o[1], o[2], o[3]), f = make_uint4(o[4], o[5], o[6], o[7]);
           uint8_t* rp = dst + row * 128;
           if (c < 4) {
@@ -228,7 +286,6 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
       }
     }
     if (!ok && lane == 0) fail();
-    if (warp == 0 && lane == 0) mbar_wait(&qfull, 0);  // the Q copy lands before the CTA leaves
   } else if (warp == 0) {
     // ---------------- TMA producer: lanes 0-15 each copy one [16][64] box of
     // a key tile (page lane & 7, head_dim half lane >> 3); lane 0 arms the
@@ -288,9 +345,12 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
   } else if (warp == 1) {
     // ---------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc_s = tc_idesc(kPaB, kPaB);                // Q, K both K-major
-      constexpr uint32_t idesc_o = tc_idesc(kPaB, kPaHD) | (1u << 16);  // V MN-major
-      bool ok = mbar_wait(&qfull, 0);
+      // Q, K both K-major; V MN-major.  int8 cache: fp16 operands (A and B
+      // of one MMA always share their type), bf16 cache: bf16
+      constexpr uint32_t f16 = KV8 ? ((1u << 7) | (1u << 10)) : 0u;
+      constexpr uint32_t idesc_s = tc_idesc(kPaB, kPaB) & ~f16;
+      constexpr uint32_t idesc_o = (tc_idesc(kPaB, kPaHD) | (1u << 16)) & ~f16;
+      bool ok = KV8 ? mbar_wait(&qconv, 0) : mbar_wait(&qfull, 0);
       const uint32_t q = smem_u32(sQ), k = smem_u32(sK), v = smem_u32(sV);
       for (int t = 0; t < nt && ok; ++t) {
         // S(t) overwrites P(t - 1): its P V has completed (in order with this thread's MMAs)
@@ -410,7 +470,7 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
             if constexpr (KV8) {
               // V scale of each key column: P V then takes the codes as they are
               const float2 vs = *reinterpret_cast<const float2*>(s_scl + (2 + (t & 1)) * kPaB + c * kPaCW + i);
-              pw[i / 2] = pa_pack(p0 * vs.x, p1 * vs.y);
+              pw[i / 2] = pa_pack_h(p0 * vs.x, p1 * vs.y);
             } else {
               pw[i / 2] = pa_pack(p0, p1);
             }
@@ -432,7 +492,8 @@ __global__ void __launch_bounds__(pa_threads<KV8>(), 2)
     }
     if (ok) {
       tc_fence_after();
-      const float inv = 1.f / l;
+      // int8 cache: P carried the V scales times 2^sigma
+      const float inv = (KV8 ? s_unscale : 1.f) / l;
       uint16_t* dst = out + ((long long)b * S + qrow) * ((long long)H * kPaHD) + (long long)h * kPaHD;
 #pragma unroll 1
       for (int c = 0; c < kPaHD / 32; ++c) {

@@ -216,7 +216,7 @@ def test_argmax_ties_lowest(fp, V):
 class Cache:
     """A paged cache built on the host (values chosen by the test), uploaded."""
 
-    def __init__(self, fp, kvq, B, T, Hkv, hd, seed, shuffle=True):
+    def __init__(self, fp, kvq, B, T, Hkv, hd, seed, shuffle=True, vs_range=(0.001, 0.03)):
         self.P, self.pps = 16, (T + 15) // 16
         self.n_pages = B * self.pps
         rng = np.random.default_rng(seed)
@@ -233,7 +233,7 @@ class Cache:
             self.k = rng.integers(-127, 128, size=shape, dtype=np.int8)
             self.v = rng.integers(-127, 128, size=shape, dtype=np.int8)
             self.ksc = synth.uniform_f32(seed, 3, shape[:3], 0.001, 0.03)
-            self.vsc = synth.uniform_f32(seed, 4, shape[:3], 0.001, 0.03)
+            self.vsc = synth.uniform_f32(seed, 4, shape[:3], *vs_range)
             self.kd, self.vd = dev(self.k), dev(self.v)
             self.ks, self.vs = dev(self.ksc), dev(self.vsc)
         self.td = dev(self.table)
@@ -287,6 +287,38 @@ def test_attention_prefill(fp, kvq, hd, H, Hkv, S):
     for b in range(B):
         ref = M.attention(qf[b], np.arange(S), c.seq("k", b, S), c.seq("v", b, S))
         assert rel_err(got[b], ref) <= TAU[0] / 2, (b, rel_err(got[b], ref))
+
+
+@pytest.mark.parametrize("vs_range", [(1e-7, 3e-7), (1e-3, 3e-2), (50.0, 400.0)])
+def test_attention_prefill_int8_value_scales(fp, vs_range):
+    """int8 cache, tcgen05 kernel (head_dim 128): P runs as fp16 carrying
+    each key's V scale times a per-CTA power of two; values far below and far
+    above the usual range of V must come out as accurately."""
+    B, S, H, Hkv, hd = 2, 300, 8, 2, 128
+    c = Cache(fp, 1, B, S + 5, Hkv, hd, seed=91, vs_range=vs_range)
+    q = synth.uniform_bf16(42, S, (B * S, H * hd), -2, 2)
+    out = empty(B * S * H * hd, np.uint16)
+    err = empty(1, np.int32)
+    fp.fp_op_attention_prefill(ptr(dev(q)), H * hd, B, S, H, c.view, ptr(out), ptr(err))
+    got = quant.bf16_to_f32(host(out, np.uint16)).reshape(B, S, H, hd)
+    qf = quant.bf16_to_f32(q).astype(np.float64).reshape(B, S, H, hd)
+    for b in range(B):
+        ref = M.attention(qf[b], np.arange(S), c.seq("k", b, S), c.seq("v", b, S))
+        assert rel_err(got[b], ref) <= TAU[0] / 2, (b, rel_err(got[b], ref))
+    assert host(err, np.int32)[0] == 0
+
+
+def test_attention_prefill_int8_q_beyond_fp16_is_reported(fp):
+    """The int8-cache tcgen05 kernel multiplies Q in fp16: a query element
+    beyond 65504 sets the error word to 3 (the runtime reports it)."""
+    B, S, H, Hkv, hd = 1, 64, 4, 2, 128
+    c = Cache(fp, 1, B, S, Hkv, hd, seed=92)
+    q = synth.uniform_bf16(43, S, (B * S, H * hd), -2, 2)
+    q[3, 17] = synth.f32_to_bf16_bits(np.array([1.0e5], np.float32))[0]
+    out = empty(B * S * H * hd, np.uint16)
+    err = empty(1, np.int32)
+    fp.fp_op_attention_prefill(ptr(dev(q)), H * hd, B, S, H, c.view, ptr(out), ptr(err))
+    assert host(err, np.int32)[0] == 3
 
 
 @pytest.mark.parametrize("kvq", [0, 1])
