@@ -96,18 +96,19 @@ def kernel_bytes(a, wq, kvq, B, ctx):
 # cached token row (units = B x context of the capture) and scales with the
 # bench's B x context.
 NCU_TRAFFIC = {
-    # profiles/dram_traffic_l70b.md: microbench cases 70b-*, one launch each
+    # profiles/dram_traffic_l70b.md and dram_traffic_l7b.md: microbench cases, one launch each
     ("l70b", "lin_gu"): {"bytes": 271997952, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
     ("l70b", "lin_down"): {"bytes": 132128000, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
     ("l70b", "lin_qkv"): {"bytes": 45146880, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
     ("l70b", "lin_o"): {"bytes": 36758528, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
-    ("l70b", "lm_head"): {"bytes": 535367936, "units": None, "src": "fp_linear.cu", "sha": "f7df17bc3111d3ac"},
+    ("l70b", "lm_head"): {"bytes": 535360768, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
     ("l70b", "attn"): {"bytes": 149525504, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
-    ("l7b", "attn"): {"bytes": 81739520, "units": 8 * 612, "src": "fp_attention.cu", "sha": "de945a405c820013"},
-    ("l7b", "lm_head"): {"bytes": 270745088, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-    ("l7b", "lin_gu"): {"bytes": 94480640, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-    ("l7b", "lin_qkv"): {"bytes": 50461184, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
-    ("l7b", "lin_o"): {"bytes": 16944384, "units": None, "src": "fp_linear.cu", "sha": "1022c24fcdb2e158"},
+    ("l7b", "attn"): {"bytes": 81390848, "units": 8 * 612, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
+    ("l7b", "lm_head"): {"bytes": 270199040, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
+    ("l7b", "lin_gu"): {"bytes": 94423040, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
+    ("l7b", "lin_qkv"): {"bytes": 50454272, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
+    ("l7b", "lin_o"): {"bytes": 16945664, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
+    ("l7b", "lin_down"): {"bytes": 45369344, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
 }
 
 
