@@ -3,7 +3,7 @@ bench times.
 
 * Llama-2-7B-, 13B- and 70B-shaped fingerprints end to end (the 70B shape:
   int4 g128 weights, int8 KV cache, GQA 64/8, batch 32, 2048-token prompts,
-  the bench's default workload): the handle is created
+  the bench's default workload; and the same with GPTQ4 weights): the handle is created
   exactly as ``bench.py`` creates it (device-side seeded weights, seed 0, unit
   norm gains, the full batch, prompt and context), prefills the full batch and
   decodes a few steps.  The oracle runs a batch-1 slice per checked sequence
@@ -16,7 +16,8 @@ bench times.
   op entry points (same kernels and plans as the runtime): the four int4
   decode linears and the LM head at M = 32 on sampled output rows, the GQA
   int8-KV decode attention at B 32 and context 2148 on sampled (sequence,
-  head) pairs, and the prefill gate+up GEMM at M = 65536 on sampled entries.
+  head) pairs, and the prefill gate+up GEMM at M = 65536 on sampled entries
+  (both prefill paths: bf16 expansion and in-kernel dequantisation).
 """
 from concurrent.futures import ThreadPoolExecutor
 
@@ -36,6 +37,8 @@ FULL = {
     "l13b": (M.Arch(2, 5120, 40, 40, 128, 13824, 32000), 2, 0, 16, 1024, 100, [5]),
     # the first and the last sequence: rows at both ends of M = 65536 in prefill
     "l70b": (M.Arch(2, 8192, 64, 8, 128, 28672, 32000), 2, 1, 32, 2048, 100, [0, 31]),
+    # the same with GPTQ4 weights (act orders drawn from the seed by fp_create)
+    "l70b_gptq4": (M.Arch(2, 8192, 64, 8, 128, 28672, 32000), 3, 1, 32, 2048, 100, [0, 31]),
 }
 N_CHECKED_DECODE = 3
 
@@ -79,7 +82,8 @@ def test_full_size_sequences_match_oracle(fp, name):
     T = S + N + 1  # the bench's context
     get = weight_getter(0, gains="ones")  # the bench's device-side init: seed 0, unit gains
     with ThreadPoolExecutor(max_workers=8) as pool:
-        w, payload = M.build_weights(arch, wq, get, map_fn=pool.map)
+        w, payload = M.build_weights(arch, wq, get, map_fn=pool.map,
+                                     act_order=lambda l, m, k: synth.act_order(0, l, m, k))
     h = fp.fp_create(arch_dict(arch), wq, kvq, B, T, seed=0, flags=fp.FP_FLAG_KEEP_HIDDEN)
     try:
         # device-side seeded weights and quantisation equal the oracle's, bit for bit
@@ -90,9 +94,11 @@ def test_full_size_sequences_match_oracle(fp, name):
                 assert np.array_equal(fp.fp_get_tensor(h, fp.FP_G_W_CODES, l, m, cdt), p["codes"].reshape(-1))
                 assert np.array_equal(fp.fp_get_tensor(h, fp.FP_G_W_SCALES, l, m, np.uint16),
                                       p["scales"].reshape(-1))
-                if wq == 2:
+                if wq in (2, 3):
                     assert np.array_equal(fp.fp_get_tensor(h, fp.FP_G_W_ZEROS, l, m, np.uint16),
                                           p["zeros"].reshape(-1))
+                if wq == 3:
+                    assert np.array_equal(fp.fp_get_tensor(h, fp.FP_G_W_PERM, l, m, np.int32), p["perm"])
         toks = synth.tokens(0, B * S, arch.vocab).reshape(B, S)
         nxt = fp.fp_prefill(h, toks)
         d = arch.hidden
@@ -212,8 +218,11 @@ def test_full_size_70b_decode_attention(fp):
     assert host(err, np.int32)[0] == 0
 
 
-def test_full_size_70b_prefill_gate_up(fp):
-    """The tcgen05 GEMM at the 70B-shaped prefill: M = 32 x 2048 rows, SwiGLU epilogue, int4 weights."""
+@pytest.mark.parametrize("scratch", [True, False])
+def test_full_size_70b_prefill_gate_up(fp, scratch):
+    """The tcgen05 GEMM at the 70B-shaped prefill: M = 32 x 2048 rows, SwiGLU
+    epilogue, int4 weights -- expanded to bf16 in the workspace, or, with no
+    workspace, dequantised inside the GEMM."""
     torch = torch_mod()
     m, n, k, wq = 32 * 2048, 2 * A70.ffn, A70.hidden, 2
     stream = 7100
@@ -222,9 +231,10 @@ def test_full_size_70b_prefill_gate_up(fp):
     fp.fp_op_init_weights(x.data_ptr(), m * k, 1, stream, 0)  # seeded bf16 activations of N(0, 0.02) shape
     nout = n // 2
     out = empty(m * nout * 2)
-    wsb = fp.fp_op_linear_workspace_bytes(wq, m, n, k)
+    wsb = fp.fp_op_linear_workspace_bytes(wq, m, n, k) if scratch else 0
     ws = empty(max(wsb, 16))
-    fp.fp_op_linear(wq, 2, x.data_ptr(), m, n, k, ptr(codes), ptr(scales), ptr(zeros), None, ptr(out), ptr(ws), wsb)
+    fp.fp_op_linear(wq, 2, x.data_ptr(), m, n, k, ptr(codes), ptr(scales), ptr(zeros), None, ptr(out),
+                    ptr(ws) if scratch else None, wsb)
     torch.cuda.synchronize()
     rng = np.random.default_rng(stream)
     mrows = np.unique(np.concatenate([[0, m - 1], rng.integers(0, m, 16)]))
