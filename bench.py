@@ -87,6 +87,14 @@ def kernel_bytes(a, wq, kvq, B, ctx):
     }
 
 
+def class_roofline(cls, kb, cls_time, launches, peak):
+    """GB/s and fraction of the HBM peak of one decode kernel class: its
+    algorithmic bytes per launch over its mean instrumented launch time."""
+    ms = cls_time[cls] / max(1, launches[cls])
+    gbs = kb[cls] / (ms * 1e-3) / 1e9 if ms > 0 else 0.0
+    return {"achieved": gbs, "frac": gbs / peak, "launch_ms": ms, "bytes_per_launch": kb[cls]}
+
+
 # ---------------------------------------------------------------- ncu traffic
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
 # decode kernels from the ncu captures summarised in profiles/ (microbench
@@ -547,6 +555,9 @@ def main():
                              "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
                              "bytes_per_launch": kb[dom], "launch_ms": per_launch_ms,
                              "traffic": ncu_traffic(dom, args.config, B, mean_ctx)},
+                # every decode kernel class the same way (instrumented launches, algorithmic bytes)
+                "roofline_by_class": {c: class_roofline(c, kb, cls_time, prof["kernel_launches"], peak)
+                                      for c in kb if prof["kernel_launches"].get(c)},
                 "gpu_launches": launches,
                 "clocks": clk.summary(),
                 "e2e": e2e,

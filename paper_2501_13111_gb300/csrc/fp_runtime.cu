@@ -378,7 +378,9 @@ int check_err_flag(fp_handle* h) {
     cudaMemsetAsync(h->err, 0, 4, h->stream);
     if (v == 2) return h->fail(FP_ERR_DEVICE_ASSERT, "a bounded wait in a pipelined kernel expired; its output is invalid");
     if (v == 3)
-      return h->fail(FP_ERR_DEVICE_ASSERT, "an activation beyond the fp16 range (|x| > 65504) reached a decode linear");
+      return h->fail(FP_ERR_DEVICE_ASSERT,
+                     "an activation beyond the fp16 range (|x| > 65504) reached a kernel that computes in fp16 "
+                     "(an int8/int4 decode linear or the int8-cache prefill attention)");
     return h->fail(FP_ERR_DEVICE_ASSERT, "a kernel met an out-of-range token id or page id and skipped it");
   }
   return FP_OK;
