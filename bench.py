@@ -109,7 +109,7 @@ NCU_TRAFFIC = {
     ("l70b", "lin_down"): {"bytes": 132128000, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
     ("l70b", "lin_qkv"): {"bytes": 45146880, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
     ("l70b", "lin_o"): {"bytes": 36758528, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
-    ("l70b", "lm_head"): {"bytes": 535360768, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
+    ("l70b", "lm_head"): {"bytes": 533600256, "units": None, "src": "fp_gemv_btc.cu", "sha": "c12906c511f2ea8b"},
     ("l70b", "attn"): {"bytes": 149525504, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
     ("l7b", "attn"): {"bytes": 81390848, "units": 8 * 612, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
     ("l7b", "lm_head"): {"bytes": 270199040, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},

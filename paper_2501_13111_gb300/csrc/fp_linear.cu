@@ -798,15 +798,12 @@ size_t linear_ws_bytes(int wquant, int M, int N, int K) {
     const size_t w = gemm_tc_ws_bytes(wquant, N, K);
     return w ? counter_bytes(0) + w : 0;
   }
-  if (!mma_ok(wquant, M, N, K)) return 0;
   size_t w = 0;
-  for (int epi : {FP_EPI_STORE, FP_EPI_RESID, FP_EPI_F32}) {
-    w = std::max(w, plan_for(wquant, epi, M, N, K).ws);
+  for (int epi : {FP_EPI_STORE, FP_EPI_RESID, FP_EPI_F32, FP_EPI_SWIGLU}) {
+    if (epi == FP_EPI_SWIGLU && N % 2 != 0) continue;
+    if (mma_ok(wquant, M, N, K)) w = std::max(w, plan_for(wquant, epi, M, N, K).ws);
     if (q4tc_ok(wquant, epi, M, N, K)) w = std::max(w, q4tc_ws_bytes(epi, M, N, K));
-  }
-  if (N % 2 == 0) {
-    w = std::max(w, plan_for(wquant, FP_EPI_SWIGLU, M, N, K).ws);
-    if (q4tc_ok(wquant, FP_EPI_SWIGLU, M, N, K)) w = std::max(w, q4tc_ws_bytes(FP_EPI_SWIGLU, M, N, K));
+    if (btc_ok(wquant, epi, M, N, K)) w = std::max(w, btc_ws_bytes(epi, M, N, K));
   }
   return w;
 }
@@ -832,6 +829,11 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
     return launch_gemm_tc(wquant, epi, x, M, N, K, codes, scales, zeros, residual, y, scratch,
                           need ? ws_bytes - counter_bytes(0) : 0, err, s);
   }
+  // bf16 weights at 17-64 tokens: the TMA-fed tcgen05 GEMV where every SM gets
+  // enough 32 KB items to hide their per-item cost (16-byte aligned x and weights)
+  if (btc_ok(wquant, epi, M, N, K) && btc_preferred(epi, N, K) && ((uintptr_t)x & 15) == 0 &&
+      ((uintptr_t)codes & 15) == 0)
+    return launch_btc(epi, x, M, N, K, codes, residual, y, ws, ws_bytes, err, s);
   // int4 at 9-64 tokens: the tensor-core path (TMA needs 16-byte aligned x and codes)
   if (q4tc_ok(wquant, epi, M, N, K) && ((uintptr_t)x & 15) == 0 && ((uintptr_t)codes & 15) == 0)
     return launch_q4tc(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, err, s);

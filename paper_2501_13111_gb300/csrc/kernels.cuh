@@ -80,6 +80,13 @@ cudaError_t launch_q4tc(int epi, const uint16_t* x, int M, int N, int K, const v
                         const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
                         int32_t* err, cudaStream_t s);
 
+// ---- bf16 decode linear at 17-64 tokens on tcgen05, TMA-fed (fp_gemv_btc.cu)
+bool btc_ok(int wquant, int epi, int M, int N, int K);
+bool btc_preferred(int epi, int N, int K);  // enough work per SM for the TMA-fed kernel
+size_t btc_ws_bytes(int epi, int M, int N, int K);
+cudaError_t launch_btc(int epi, const uint16_t* x, int M, int N, int K, const void* w, const uint16_t* residual,
+                       void* y, void* ws, size_t ws_bytes, int32_t* err, cudaStream_t s);
+
 // ---- prefill GEMM on tcgen05 (fp_gemm_tc.cu)
 bool gemm_tc_ok(int M, int N, int K);
 size_t gemm_tc_ws_bytes(int wquant, int N, int K);

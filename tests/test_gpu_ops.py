@@ -501,3 +501,33 @@ def test_prefill_linear_in_bands_of_columns(fp, scratch, wq, m, n, k, epi):
     elif epi == 2:
         y = M.silu(y[:, :nout]) * y[:, nout:]
     assert rel_err(got, y) <= TAU[wq] / 4, rel_err(got, y)
+
+
+@pytest.mark.parametrize("m", [17, 32, 33, 64])
+@pytest.mark.parametrize("epi", [0, 1, 2, 3])
+def test_linear_bf16_tensor_core(fp, m, epi):
+    """bf16 weights at 17-64 tokens with enough work per SM run on the
+    TMA-fed tcgen05 GEMV (the LM head's kernel): ragged last row tile (N not a
+    multiple of 128) and a K tail (half of the last 128-k item past K); output
+    columns checked on a sample, the first and the last included."""
+    n, k = (2 * 16424, 4160) if epi == 2 else (16424, 8256)
+    w = synth.weight_bf16(51, 0, 1, (n, k))
+    x = synth.uniform_bf16(52, m, (m, k), -2.0, 2.0)
+    nout = n // 2 if epi == 2 else n
+    r = synth.uniform_bf16(53, m, (m, nout), -1.0, 1.0)
+    out = empty(m * nout * (4 if epi == 3 else 2))
+    ws_b = fp.fp_op_linear_workspace_bytes(0, m, n, k)
+    ws = empty(max(ws_b, 16))
+    fp.fp_op_linear(0, epi, ptr(dev(x)), m, n, k, ptr(dev(w)), None, None, ptr(dev(r)), ptr(out), ptr(ws), ws_b)
+    got = host(out, np.float32) if epi == 3 else quant.bf16_to_f32(host(out, np.uint16))
+    got = got.reshape(m, nout).astype(np.float64)
+    cols = np.unique(np.concatenate([[0, nout - 1], np.random.default_rng(m + epi).integers(0, nout, 96)]))
+    xf = quant.bf16_to_f32(x).astype(np.float64)
+    wf = lambda rows: quant.bf16_to_f32(w[rows]).astype(np.float64)
+    if epi == 2:
+        ref = M.silu(xf @ wf(cols).T) * (xf @ wf(cols + nout).T)
+    else:
+        ref = xf @ wf(cols).T
+        if epi == 1:
+            ref = ref + quant.bf16_to_f32(r).astype(np.float64)[:, cols]
+    assert rel_err(got[:, cols], ref) <= TAU[0] / 4, (m, epi, rel_err(got[:, cols], ref))
