@@ -105,18 +105,18 @@ def class_roofline(cls, kb, cls_time, launches, peak):
 # bench's B x context.
 NCU_TRAFFIC = {
     # profiles/dram_traffic_l70b.md and dram_traffic_l7b.md: microbench cases, one launch each
-    ("l70b", "lin_gu"): {"bytes": 271997952, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
-    ("l70b", "lin_down"): {"bytes": 132128000, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
-    ("l70b", "lin_qkv"): {"bytes": 45146880, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
-    ("l70b", "lin_o"): {"bytes": 36758528, "units": None, "src": "fp_gemv_tc.cu", "sha": "331527d441d4b150"},
-    ("l70b", "lm_head"): {"bytes": 533600256, "units": None, "src": "fp_gemv_btc.cu", "sha": "c12906c511f2ea8b"},
+    ("l70b", "lin_gu"): {"bytes": 273308928, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
+    ("l70b", "lin_down"): {"bytes": 130883584, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
+    ("l70b", "lin_qkv"): {"bytes": 45146368, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
+    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
+    ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "bd39d79e47b0ba01"},
     ("l70b", "attn"): {"bytes": 149525504, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
     ("l7b", "attn"): {"bytes": 81390848, "units": 8 * 612, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
-    ("l7b", "lm_head"): {"bytes": 270199040, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
-    ("l7b", "lin_gu"): {"bytes": 94423040, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
-    ("l7b", "lin_qkv"): {"bytes": 50454272, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
-    ("l7b", "lin_o"): {"bytes": 16945664, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
-    ("l7b", "lin_down"): {"bytes": 45369344, "units": None, "src": "fp_linear.cu", "sha": "3811218390a7db20"},
+    ("l7b", "lm_head"): {"bytes": 270125824, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
+    ("l7b", "lin_gu"): {"bytes": 94427904, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
+    ("l7b", "lin_qkv"): {"bytes": 50466304, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
+    ("l7b", "lin_o"): {"bytes": 16945920, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
+    ("l7b", "lin_down"): {"bytes": 45368576, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
 }
 
 

@@ -201,10 +201,14 @@ __global__ void __launch_bounds__(kBtThreads, 1)
       if (lane == 0) mbar_arrive(&tempty[buf]);
 
       const int row = b * kBtRows + lr;
-      auto finish = [&](int m, float v, float u) {
+      // r: the residual R[m][row], read before any store (R may be Y itself)
+      auto resid = [&](int m) {
+        return (EPI == FP_EPI_RESID && m < M && row < Nout) ? bf2f(R[(long long)m * Nout + row]) : 0.f;
+      };
+      auto finish = [&](int m, float v, float u, float r) {
         const long long o = (long long)m * Nout + row;
         if constexpr (EPI == FP_EPI_STORE) ((uint16_t*)Y)[o] = f2bf(v);
-        else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(bf2f(R[o]) + v);
+        else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(r + v);
         else if constexpr (EPI == FP_EPI_SWIGLU) ((uint16_t*)Y)[o] = f2bf(silu(v) * u);
         else ((float*)Y)[o] = v;
       };
@@ -212,8 +216,15 @@ __global__ void __launch_bounds__(kBtThreads, 1)
       const long long c1 = bt_cta_of((long long)(b + 1) * S - 1, C, total);
       if (c0 == c1) {
 #pragma unroll
-        for (int i = 0; i < MT; ++i)
-          if (i < M && row < Nout) finish(i, __uint_as_float(dv[0][i]), __uint_as_float(dv[NR - 1][i]));
+        for (int i0 = 0; i0 < MT; i0 += 8) {
+          float rv[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) rv[i] = resid(i0 + i);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (i0 + i < M && row < Nout)
+              finish(i0 + i, __uint_as_float(dv[0][i0 + i]), __uint_as_float(dv[NR - 1][i0 + i]), rv[i]);
+        }
         continue;
       }
       // partial slot b + c: distinct for every (row tile, CTA) pair that meets
@@ -231,15 +242,31 @@ __global__ void __launch_bounds__(kBtThreads, 1)
       t = __shfl_sync(0xffffffffu, t, 0);
       if (t != (unsigned)(c1 - c0)) continue;
       __threadfence();
+      // the sum over the CTAs in CTA order (deterministic), eight tokens' loads
+      // in flight per CTA rather than one
       const int cnt = (int)(c1 - c0) + 1;
-      for (int i = 0; i < M; ++i) {
-        const float* p0 = ws + (size_t)(b + c0) * slot + (size_t)i * NR * kBtRows + lr;
-        float v = 0.f, u = 0.f;
+      const float* p0 = ws + (size_t)(b + c0) * slot + lr;
+#pragma unroll
+      for (int i0 = 0; i0 < MT; i0 += 8) {
+        if (i0 >= M) break;
+        float v[8], u[8], rv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = u[i] = 0.f, rv[i] = resid(i0 + i);
         for (int cc = 0; cc < cnt; ++cc) {
-          v += __ldcg(p0 + (size_t)cc * slot);
-          if (NR == 2) u += __ldcg(p0 + (size_t)cc * slot + kBtRows);
+          const float* pc = p0 + (size_t)cc * slot;
+          float t[8], t2[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const bool in = i0 + i < M;
+            t[i] = in ? __ldcg(pc + (size_t)(i0 + i) * NR * kBtRows) : 0.f;
+            t2[i] = (NR == 2 && in) ? __ldcg(pc + (size_t)(i0 + i) * NR * kBtRows + kBtRows) : 0.f;
+          }
+#pragma unroll
+          for (int i = 0; i < 8; ++i) v[i] += t[i], u[i] += t2[i];
         }
-        if (row < Nout) finish(i, v, u);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if (i0 + i < M && row < Nout) finish(i0 + i, v[i], u[i], rv[i]);
       }
       if (lane == 0) counters[b * 4 + ew] = 0u;
     }

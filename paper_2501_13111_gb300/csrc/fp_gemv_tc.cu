@@ -9,25 +9,29 @@
 // lane each) and the tokens the N dimension of tcgen05.mma (M 128, N =
 // tokens rounded up to 32 or 64, K 16):
 //   warps 0-15  dequantise, in two teams of eight that take alternate
-//               128-k groups: warp w owns TMEM lanes 32 (w % 4) .. +31 (one
-//               weight row per thread) and half of a group (SwiGLU: a whole
-//               group of the gate or the up tile).  Each thread streams its
+//               items (two consecutive 128-k groups where K allows, else one;
+//               SwiGLU: one group of the gate and of the up tile): warp w
+//               owns TMEM lanes 32 (w % 4) .. +31 (one weight row per thread)
+//               and one group of the item (else half of it).  Each thread streams its
 //               own codes through a private cp.async ring in shared memory
 //               (no cross-warp handshake),
 //               forms bf16((q - z) s) -- exactly the prefill expansion --
 //               and stores them into an A slot of TMEM (tcgen05.st, two K
 //               elements per 32-bit column); afull / aempty hand the slots
 //               to the MMA thread and back;
-//   warp 16     TMA producer of x ([N][128] bf16 per group, two
+//   warp 16     TMA producer of x ([N][128] bf16 per group as two
 //               128-byte-swizzled boxes, rows past M zero-filled) into a ring
-//               (xfull / xempty, freed by the MMAs);
+//               whose stage a goes with A slot a: afull[a] completes when the
+//               team's warps have stored the slot and the x bytes have
+//               landed, and one commit of the MMAs frees both (aempty[a]), so
+//               the MMA thread waits once and commits once per item;
 //   warp 17     allocates 512 TMEM columns and issues the MMAs (A from TMEM,
 //               B = x from shared memory) into fp32 TMEM accumulators.
 // MMAs (M 128, N <= 64, K 16) into one accumulator follow each other at
 // about 50 cycles, far above their math (N / 2 cycles), while MMAs into
 // different accumulators overlap: the k-steps of each matrix are spread
 // round-robin over 2-4 accumulators ("chains"), summed in the epilogue.
-// The (row tile, group) pairs are split into equal contiguous ranges, one
+// The (row tile, item) pairs are split into equal contiguous ranges, one
 // per SM (stream-K, as the CUDA-core GEMV): a CTA whose range covers a whole
 // row tile runs the epilogue itself; otherwise each of its sixteen warps
 // writes fp32 partials of its 32 rows x a quarter of the tokens, and the
@@ -53,22 +57,31 @@ constexpr uint32_t kQ4TmemCols = 512;
 constexpr int kQ4Rows = 128;
 constexpr int kQ4MinSmem = 116 * 1024;  // above half an SM: one CTA (and one TMEM owner) per SM
 
-template <int MT, int NR>
+// An item is GPI consecutive 128-k groups of one row tile (of the gate and
+// the up tile with SwiGLU).  Without SwiGLU two groups per item (K a multiple
+// of 256) halve the hand-offs per byte: each item then carries 16 KB of
+// codes, as a SwiGLU item does.
+template <int MT, int NR, int GPI>
 struct Q4Geom {
-  // each thread takes every other group: a whole group of its row (SwiGLU:
-  // of the gate or the up row), otherwise half of one
-  static constexpr int kChunks = NR == 2 ? 4 : 2;        // 16-byte code chunks per thread and group
+  static_assert(GPI == 1 || NR == 1, "SwiGLU items hold one group of each matrix");
+  // each thread takes every other item: a whole group of its row (SwiGLU: of
+  // the gate or the up row; GPI 2: the first or the second group), otherwise
+  // half of one
+  static constexpr int kChunks = (NR == 2 || GPI == 2) ? 4 : 2;  // 16-byte code chunks per thread and item
   static constexpr int kCodeBytes = kQ4DeqWarps * 32 * kChunks * 16;  // one ring stage, all threads
-  static constexpr int kXBytes = MT * 256;               // x [MT][128] bf16 as two [MT][64] boxes
+  static constexpr int kXBytes = GPI * MT * 256;         // x [MT][128 GPI] bf16 as [MT][64] boxes
   // independent accumulation chains per matrix
   static constexpr int kChains = MT == 64 ? 2 / NR : 4 / NR;
   static constexpr int kDCols = NR * kChains * MT;       // fp32 accumulators
-  static constexpr int kACols = NR * 64;                 // one group of bf16 pairs per matrix
+  static constexpr int kACols = NR * GPI * 64;           // the item's bf16 pairs
   static constexpr int kASlots = std::min(6, ((int)kQ4TmemCols - kDCols) / kACols);
-  static constexpr int kXStages = MT == 64 ? 4 : 6;
+  // x stage a travels with A slot a: one barrier per item says both are ready
+  // and one commit frees both
+  static constexpr int kXStages = kASlots;
   static constexpr int kSmem = kQ4CodeStages * kCodeBytes + kXStages * kXBytes + 1024;
   static_assert(kASlots >= 2 && kDCols + kASlots * kACols <= (int)kQ4TmemCols, "TMEM budget");
   static_assert(kCodeBytes % 1024 == 0 && kXBytes % 1024 == 0, "x stages stay 1024-byte aligned");
+  static_assert(kSmem <= 227 * 1024, "shared memory");
 };
 
 // 16-byte asynchronous global -> shared copy (L2 only) and its group fences.
@@ -123,18 +136,19 @@ FP_DEV void deq_word(uint32_t w, uint32_t zz, uint32_t ss, uint32_t* out) {
 
 FP_DEV long long q4_cta_of(long long i, long long C, long long total) { return ((i + 1) * C - 1) / total; }
 
-template <int MT, int EPI>
+template <int MT, int EPI, int GPI>
 __global__ void __launch_bounds__(kQ4Threads, 1)
     gemv_q4tc_kernel(const __grid_constant__ CUtensorMap map_x, const uint8_t* __restrict__ codes, int M, int N,
                      const uint16_t* __restrict__ scales, const uint16_t* __restrict__ zeros, const uint16_t* R,
                      void* Y, long long total, int S, int V, float* __restrict__ ws, unsigned* __restrict__ counters,
                      int32_t* err) {
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
-  using G = Q4Geom<MT, NR>;
+  using G = Q4Geom<MT, NR, GPI>;
   constexpr int CS = kQ4CodeStages, XS = G::kXStages, NA = G::kASlots, MQ = MT / 4, DW = kQ4DeqWarps;
   constexpr int NCH = G::kChains, CK = G::kChunks;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
-  __shared__ uint64_t xfull[XS], xempty[XS], afull[NA], aempty[NA], dfull, dempty, mma_done;
+  static_assert(XS == NA, "x stages and A slots share their barriers");
+  __shared__ uint64_t afull[NA], aempty[NA], dfull, dempty, mma_done;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_word;
   volatile int* abort_flag = &abort_word;
@@ -146,6 +160,7 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
   const long long C = gridDim.x, c = blockIdx.x;
   const long long begin = c * total / C, end = (c + 1) * total / C;
   const int L = (int)(end - begin);
+  const int SI = S / GPI;  // items per row tile
   auto fail = [&]() {
     *abort_flag = 1;
     if (err) atomicExch(err, 2);
@@ -153,13 +168,11 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
 
   pdl_trigger();
   if (threadIdx.x == 0) {
-    for (int s = 0; s < XS; ++s) {
-      mbar_init(&xfull[s], 1);   // producer's expect_tx; completes with the bytes
-      mbar_init(&xempty[s], kQ4MmaWarps);  // tcgen05.commit of the MMAs that read x
-    }
     for (int a = 0; a < NA; ++a) {
-      mbar_init(&afull[a], DW / 2);  // the eight warps of the group's team stored its A columns
-      mbar_init(&aempty[a], kQ4MmaWarps);  // tcgen05.commit of the MMAs that read the slot
+      // the eight warps of the group's team stored its A columns, and the x
+      // producer's expect_tx, completed by the bytes of the group's x
+      mbar_init(&afull[a], DW / 2 + 1);
+      mbar_init(&aempty[a], kQ4MmaWarps);  // tcgen05.commit of the MMAs that read slot and stage
     }
     mbar_init(&dfull, kQ4MmaWarps);
     mbar_init(&dempty, DW);
@@ -183,21 +196,23 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
     if (lane == 0) {
       pdl_wait();  // x is the previous kernel's output
       int issued = 0;
-      int g = (int)(begin % S);
-      for (int q = 0; q < L; ++q, g = g + 1 == S ? 0 : g + 1) {
+      int g = (int)(begin % SI);
+      for (int q = 0; q < L; ++q, g = g + 1 == SI ? 0 : g + 1) {
         const int s = q % XS;
-        if (q >= XS && (!mbar_wait_sleep(&xempty[s], ((q / XS) & 1) ^ 1) || *abort_flag)) {
+        if (q >= XS && (!mbar_wait_sleep(&aempty[s], ((q / XS) & 1) ^ 1) || *abort_flag)) {
           fail();
           break;
         }
         uint8_t* xs = x_ring + s * G::kXBytes;
-        mbar_expect_tx(&xfull[s], G::kXBytes);
-        tma_load_2d(xs, &map_x, g * 128, 0, &xfull[s]);
-        tma_load_2d(xs + MT * 128, &map_x, g * 128 + 64, 0, &xfull[s]);
+        mbar_expect_tx(&afull[s], G::kXBytes);
+#pragma unroll
+        for (int bx = 0; bx < 2 * GPI; ++bx) tma_load_2d(xs + bx * MT * 128, &map_x, g * GPI * 128 + bx * 64, 0, &afull[s]);
         issued = q + 1;
       }
-      // copies still in flight land before the CTA leaves (their stages are its shared memory)
-      for (int j = max(0, issued - XS); j < issued; ++j) mbar_wait(&xfull[j % XS], (j / XS) & 1);
+      // copies still in flight land before the CTA leaves (their stages are its
+      // shared memory); after an abort the phase may never complete, and the
+      // bounded wait then outlasts the copies
+      for (int j = max(0, issued - XS); j < issued; ++j) mbar_wait(&afull[j % XS], (j / XS) & 1);
     }
   } else if (warp > DW) {
     // ---------------- MMA issuers: SwiGLU, one per matrix; otherwise even / odd k-steps
@@ -206,13 +221,12 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       constexpr uint32_t idesc = tc_idesc(kQ4Rows, MT);
       int seg = 0;
       bool ok = true;
-      int g = (int)(begin % S);
-      for (int q = 0; q < L; ++q, g = g + 1 == S ? 0 : g + 1) {
-        const bool first = q == 0 || g == 0, last = g == S - 1 || q == L - 1;
+      int g = (int)(begin % SI);
+      for (int q = 0; q < L; ++q, g = g + 1 == SI ? 0 : g + 1) {
+        const bool first = q == 0 || g == 0, last = g == SI - 1 || q == L - 1;
         const int s = q % XS, a = q % NA;
-        if (first && seg > 0) ok = mbar_wait_sleep(&dempty, (seg - 1) & 1);  // the epilogue has read D
-        ok = ok && mbar_wait_sleep(&xfull[s], (q / XS) & 1) && mbar_wait_sleep(&afull[a], (q / NA) & 1) &&
-             !*abort_flag;
+        if (first && seg > 0) ok = mbar_wait(&dempty, (seg - 1) & 1);  // the epilogue has read D
+        ok = ok && mbar_wait(&afull[a], (q / NA) & 1) && !*abort_flag;  // A slot and x stage
         if (!ok) break;
         tc_fence_after();
         const uint64_t xd = sdesc(smem_u32(x_ring + s * G::kXBytes));
@@ -221,15 +235,15 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
         // MMAs of one issuer never share an accumulator, and the two issuers'
         // chains are disjoint
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
+        for (int kk = 0; kk < 8 * GPI; ++kk) {
           const int r = NR == 2 ? mw : 0;
           if (NR == 1 && (kk & 1) != mw) continue;
-          // descriptor start addresses count 16-byte units
+          // descriptor start addresses count 16-byte units; k-step kk reads A
+          // columns 8 kk .. +7 (of matrix r) and x box kk / 4
           tc_mma_ts(tmem + (r * NCH + kk % NCH) * MT, ta + r * 64 + kk * 8,
                     xd + (uint64_t)(((kk >> 2) * MT * 128 + (kk & 3) * 32) >> 4), idesc, (first && kk < NCH) ? 0u : 1u);
         }
-        tc_commit(&xempty[s]);  // x of stage s has been read
-        tc_commit(&aempty[a]);  // A slot a has been read
+        tc_commit(&aempty[a]);  // A slot a and x stage a have been read
         if (last) {
           tc_commit(&dfull);
           ++seg;
@@ -242,38 +256,40 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
     }
   } else {
     // ---------------- dequantise (+ epilogue)
-    // two teams of eight warps take alternate groups, so one team computes
+    // two teams of eight warps take alternate items, so one team computes
     // while the other waits; within a team warp w owns TMEM lanes
-    // 32 (w % 4) .. +31 and, SwiGLU, the gate or the up rows, otherwise the
-    // first or second half of the group
+    // 32 (w % 4) .. +31 and, SwiGLU, the gate or the up rows, with two groups
+    // per item the first or the second group, otherwise the first or second
+    // half of the group
     const int qd = warp & 3, team = warp >> 3, half = (warp >> 2) & 1, lr = qd * 32 + lane;
     const int pt = warp >> 2;  // epilogue: tokens [pt MQ, (pt + 1) MQ)
     const int rm = NR == 2 ? half : 0;
-    const int cbase = NR == 2 ? 0 : 2 * half;  // first 16-byte chunk of the row's 64 bytes
-    const int acol = NR == 2 ? rm * 64 : half * 32;
+    const int gsel = GPI == 2 ? half : 0;                    // this warp's group of the item
+    const int cbase = (NR == 1 && GPI == 1) ? 2 * half : 0;  // first 16-byte chunk of the group's 64 bytes
+    const int acol = NR == 2 ? rm * 64 : GPI == 2 ? half * 64 : half * 32;
     const uint32_t lane_base = tmem + ((uint32_t)(qd * 32) << 16);
     const long long row_bytes = (long long)S * 64;
 
-    // ---- this thread's code ring: its n-th own group (pair team + 2 n) in stage
+    // ---- this thread's code ring: its n-th own item (team + 2 n) in stage
     // n % CS, chunk i at [stage][i][thread] (a warp's loads of one chunk are
     // 512 contiguous bytes)
     uint8_t* my_ring = code_ring + (size_t)threadIdx.x * 16;
-    const int own = (L - team + 1) / 2;  // groups this team takes
-    int ib = (int)((begin + team) / S), ig = (int)((begin + team) % S);  // (row tile, group) of the next copy
+    const int own = (L - team + 1) / 2;  // items this team takes
+    int ib = (int)((begin + team) / SI), ig = (int)((begin + team) % SI);  // (row tile, item) of the next copy
     const uint8_t* src = nullptr;
     auto set_src = [&]() {
       const long long rr = min(ib * kQ4Rows + lr, Nout - 1) + rm * Nout;
-      src = codes + rr * row_bytes + cbase * 16;
+      src = codes + rr * row_bytes + gsel * 64 + cbase * 16;
     };
     if (own > 0) set_src();
     auto issue = [&](int n) {  // called for n = 0, 1, 2, ... in order
       if (n < own) {
         uint8_t* d = my_ring + (size_t)(n % CS) * G::kCodeBytes;
 #pragma unroll
-        for (int i = 0; i < CK; ++i) q4_cp16(d + i * (DW * 32 * 16), src + (long long)ig * 64 + i * 16);
+        for (int i = 0; i < CK; ++i) q4_cp16(d + i * (DW * 32 * 16), src + (long long)ig * (GPI * 64) + i * 16);
         ig += 2;
-        if (ig >= S) {
-          while (ig >= S) ig -= S, ++ib;
+        if (ig >= SI) {
+          while (ig >= SI) ig -= SI, ++ib;
           if (n + 1 < own) set_src();
         }
       }
@@ -283,56 +299,52 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
 #pragma unroll 1
     for (int n = 0; n < CS - 1; ++n) issue(n);
 
-    // scales and zeros of the row, V groups per load, one chunk ahead (S % V == 0,
-    // so a chunk never crosses a row tile)
+    // scales and zeros of the row, V groups (VI items) per load, one chunk
+    // ahead (S % V == 0, so a chunk never crosses a row tile)
+    const int VI = V / GPI;
     uint4 s_cur, z_cur, s_nxt = make_uint4(0u, 0u, 0u, 0u), z_nxt = s_nxt;
-    auto load_chunk = [&](int bb, int g0, uint4& sv, uint4& zv) {
-      const long long idx = (long long)(min(bb * kQ4Rows + lr, Nout - 1) + rm * Nout) * S + g0;
+    auto load_chunk = [&](int bb, int g0, uint4& sv, uint4& zv) {  // g0: first item of the chunk
+      const long long idx = (long long)(min(bb * kQ4Rows + lr, Nout - 1) + rm * Nout) * S + (long long)g0 * GPI;
       sv = ld_groups(scales + idx, V);
       zv = ld_groups(zeros + idx, V);
     };
-    // (row tile, group) of the current pair and its place j in the chunk of V
-    // groups, advanced without divisions
-    int b = (int)(begin / S), g = (int)(begin % S), j = g % V;
+    // (row tile, item) of the current item and its place j in the chunk of VI
+    // items, advanced without divisions
+    int b = (int)(begin / SI), g = (int)(begin % SI), j = g % VI;
     load_chunk(b, g - j, s_cur, z_cur);
-    auto prefetch_next = [&](long long p_next, int bb, int g0) {  // the chunk starting at pair p_next
-      if (g0 == S) g0 = 0, ++bb;
+    auto prefetch_next = [&](long long p_next, int bb, int g0) {  // the chunk starting at item p_next
+      if (g0 == SI) g0 = 0, ++bb;
       if (p_next < end) load_chunk(bb, g0, s_nxt, z_nxt);
     };
-    prefetch_next(begin - j + V, b, g - j + V);
+    prefetch_next(begin - j + VI, b, g - j + VI);
     pdl_wait();
     int seg = 0;
     for (int q = 0; q < L; ++q) {
       const long long p = begin + q;
       if (q > 0) {
-        if (++g == S) g = 0, ++b;
-        if (++j == V) {
+        if (++g == SI) g = 0, ++b;
+        if (++j == VI) {
           j = 0;
           s_cur = s_nxt;
           z_cur = z_nxt;
-          prefetch_next(p + V, b, g + V);
+          prefetch_next(p + VI, b, g + VI);
         }
       }
-      const bool last = g == S - 1 || q == L - 1;
+      const bool last = g == SI - 1 || q == L - 1;
       if ((q & 1) == team) {
         const int n = q >> 1, a = q % NA;
-        q4_wait<CS - 2>();  // this thread's copies of its n-th group have landed
+        q4_wait<CS - 2>();  // this thread's copies of its n-th item have landed
         uint4 wv[CK];
 #pragma unroll
         for (int i = 0; i < CK; ++i)
           wv[i] = *reinterpret_cast<const uint4*>(my_ring + (size_t)(n % CS) * G::kCodeBytes + i * (DW * 32 * 16));
-        issue(n + CS - 1);  // refills the stage read one own group ago
+        issue(n + CS - 1);  // refills the stage read one own item ago
 
-        const uint32_t sb = bf16_at(s_cur, j);
-        const uint32_t zb = f2bf(128.f + bf2f((uint16_t)bf16_at(z_cur, j)));
+        const uint32_t sb = bf16_at(s_cur, j * GPI + gsel);
+        const uint32_t zb = f2bf(128.f + bf2f((uint16_t)bf16_at(z_cur, j * GPI + gsel)));
         const uint32_t ss = sb | (sb << 16), zz = zb | (zb << 16);
-        bool ok = mbar_wait_sleep(&aempty[a], ((q / NA) & 1) ^ 1);
-        if (!__all_sync(0xffffffffu, ok) || __any_sync(0xffffffffu, *abort_flag != 0)) {
-          if (lane == 0) fail();
-          break;
-        }
-        tc_fence_after();
         const uint32_t ta = lane_base + G::kDCols + a * G::kACols + acol;
+        bool ok = true;
 #pragma unroll
         for (int h2 = 0; h2 < CK / 2; ++h2) {  // 32 columns (two chunks) per store
           uint32_t av[32];
@@ -344,7 +356,17 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
             deq_word(w.z, zz, ss, av + i * 16 + 8);
             deq_word(w.w, zz, ss, av + i * 16 + 12);
           }
+          if (h2 == 0) {  // the first columns are converted while the slot drains
+            ok = mbar_wait_sleep(&aempty[a], ((q / NA) & 1) ^ 1);
+            ok = __all_sync(0xffffffffu, ok) && !__any_sync(0xffffffffu, *abort_flag != 0);
+            if (!ok) break;
+            tc_fence_after();
+          }
           tc_st32(ta + h2 * 32, av);
+        }
+        if (!ok) {
+          if (lane == 0) fail();
+          break;
         }
         tc_wait_st();
         tc_fence_before();
@@ -379,19 +401,30 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       ++seg;
 
       const int row = b * kQ4Rows + lr;
-      auto finish = [&](int m, float v, float u) {
+      // r: the residual R[m][row], read before any store (R may be Y itself)
+      auto resid = [&](int m) {
+        return (EPI == FP_EPI_RESID && m < M && row < Nout) ? bf2f(R[(long long)m * Nout + row]) : 0.f;
+      };
+      auto finish = [&](int m, float v, float u, float r) {
         const long long o = (long long)m * Nout + row;
         if constexpr (EPI == FP_EPI_STORE) ((uint16_t*)Y)[o] = f2bf(v);
-        else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(bf2f(R[o]) + v);
+        else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(r + v);
         else if constexpr (EPI == FP_EPI_SWIGLU) ((uint16_t*)Y)[o] = f2bf(silu(v) * u);
         else ((float*)Y)[o] = v;
       };
-      const long long c0 = q4_cta_of((long long)b * S, C, total);
-      const long long c1 = q4_cta_of((long long)(b + 1) * S - 1, C, total);
+      const long long c0 = q4_cta_of((long long)b * SI, C, total);
+      const long long c1 = q4_cta_of((long long)(b + 1) * SI - 1, C, total);
       if (c0 == c1) {
 #pragma unroll
-        for (int i = 0; i < MQ; ++i)
-          if (m0 + i < M && row < Nout) finish(m0 + i, __uint_as_float(dv[0][i]), __uint_as_float(dv[NR - 1][i]));
+        for (int i0 = 0; i0 < MQ; i0 += 8) {
+          float rv[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) rv[i] = resid(m0 + i0 + i);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (m0 + i0 + i < M && row < Nout)
+              finish(m0 + i0 + i, __uint_as_float(dv[0][i0 + i]), __uint_as_float(dv[NR - 1][i0 + i]), rv[i]);
+        }
         continue;
       }
       // partial slot b + c: distinct for every (row tile, CTA) pair that meets
@@ -409,15 +442,30 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       t = __shfl_sync(0xffffffffu, t, 0);
       if (t != (unsigned)(c1 - c0)) continue;
       __threadfence();
+      // the sum over the CTAs in CTA order (deterministic), eight tokens' loads
+      // in flight per CTA rather than one
       const int cnt = (int)(c1 - c0) + 1;
-      for (int i = 0; i < MQ && m0 + i < M; ++i) {
-        const float* p0 = ws + (size_t)(b + c0) * slot + (size_t)(m0 + i) * NR * kQ4Rows + lr;
-        float v = 0.f, u = 0.f;
+      const float* p0 = ws + (size_t)(b + c0) * slot + (size_t)m0 * NR * kQ4Rows + lr;
+#pragma unroll
+      for (int i0 = 0; i0 < MQ; i0 += 8) {
+        float v[8], u[8], rv[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[i] = u[i] = 0.f, rv[i] = resid(m0 + i0 + i);
         for (int cc = 0; cc < cnt; ++cc) {
-          v += __ldcg(p0 + (size_t)cc * slot);
-          if (NR == 2) u += __ldcg(p0 + (size_t)cc * slot + kQ4Rows);
+          const float* pc = p0 + (size_t)cc * slot;
+          float t[8], t2[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const bool in = m0 + i0 + i < M;
+            t[i] = in ? __ldcg(pc + (size_t)(i0 + i) * NR * kQ4Rows) : 0.f;
+            t2[i] = (NR == 2 && in) ? __ldcg(pc + (size_t)(i0 + i) * NR * kQ4Rows + kQ4Rows) : 0.f;
+          }
+#pragma unroll
+          for (int i = 0; i < 8; ++i) v[i] += t[i], u[i] += t2[i];
         }
-        if (row < Nout) finish(m0 + i, v, u);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          if (m0 + i0 + i < M && row < Nout) finish(m0 + i0 + i, v[i], u[i], rv[i]);
       }
       if (lane == 0) counters[b * DW + warp] = 0u;
     }
@@ -462,19 +510,19 @@ size_t q4tc_ws_bytes(int epi, int M, int N, int K) {
   return (size_t)kLinTicketSlots * 4 + (size_t)(blocks + ctas) * M * nr * kQ4Rows * 4;
 }
 
-template <int MT, int EPI>
+template <int MT, int EPI, int GPI>
 static cudaError_t launch_q4_t(const uint8_t* codes, const CUtensorMap& mx, int M, int N, int K,
                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* Y, void* ws,
                                int32_t* err, cudaStream_t s) {
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
-  auto kern = gemv_q4tc_kernel<MT, EPI>;
-  const int smem = std::max(Q4Geom<MT, NR>::kSmem, kQ4MinSmem);
+  auto kern = gemv_q4tc_kernel<MT, EPI, GPI>;
+  const int smem = std::max(Q4Geom<MT, NR, GPI>::kSmem, kQ4MinSmem);
   static std::atomic<unsigned long long> attr{0};
   FP_CUDA_TRY(smem_limit_once(kern, smem, &attr));
   const int nout = NR == 2 ? N / 2 : N;
   const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
   const int S = K / 128;
-  const long long total = blocks * S;
+  const long long total = blocks * (S / GPI);  // items
   const int ctas = (int)std::min<long long>(total, q4_sms());
   unsigned* counters = (unsigned*)ws;
   float* part = (float*)((char*)ws + (size_t)kLinTicketSlots * 4);
@@ -486,11 +534,19 @@ template <int MT>
 static cudaError_t launch_q4_m(int epi, const uint8_t* mw, const CUtensorMap& mx, int M, int N, int K,
                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* Y, void* ws,
                                int32_t* err, cudaStream_t s) {
+  // two groups per item where K allows (SwiGLU items already carry two)
+  const bool two = (K / 128) % 2 == 0;
   switch (epi) {
-    case FP_EPI_STORE: return launch_q4_t<MT, FP_EPI_STORE>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
-    case FP_EPI_RESID: return launch_q4_t<MT, FP_EPI_RESID>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
-    case FP_EPI_SWIGLU: return launch_q4_t<MT, FP_EPI_SWIGLU>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
-    default: return launch_q4_t<MT, FP_EPI_F32>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    case FP_EPI_STORE:
+      return two ? launch_q4_t<MT, FP_EPI_STORE, 2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
+                 : launch_q4_t<MT, FP_EPI_STORE, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    case FP_EPI_RESID:
+      return two ? launch_q4_t<MT, FP_EPI_RESID, 2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
+                 : launch_q4_t<MT, FP_EPI_RESID, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    case FP_EPI_SWIGLU: return launch_q4_t<MT, FP_EPI_SWIGLU, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    default:
+      return two ? launch_q4_t<MT, FP_EPI_F32, 2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
+                 : launch_q4_t<MT, FP_EPI_F32, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
   }
 }
 
