@@ -546,7 +546,8 @@ __global__ void __launch_bounds__(kD8Warps * 32) attn_decode_i8_kernel(
   constexpr int HD = 128;
   extern __shared__ __align__(16) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
-  pdl_trigger();
+  // no early trigger: the linear after it takes whole SMs, and launched early
+  // its CTAs would sit beside these and stream weights while they stream the cache
   pdl_wait();
   const int Hkv = kv.n_kv_heads;
   const int b = blockIdx.x / Hkv, kvh = blockIdx.x % Hkv;

@@ -233,10 +233,14 @@ cudaError_t launch_argmax(const float* logits, int M, int V, int32_t* out, cudaS
 // rounded to bf16.  Keys and values go to the paged cache; with an int8
 // cache each (token, KV head) row is quantised: s = fp32(max|x| / 127),
 // q = clamp(rint(fp32(x / s)), -127, 127).
+//
+// No early trigger: the attention after it is launched once this kernel has
+// finished, when the linear before it has left every SM, so that its CTAs
+// spread over all SMs (launched early, they piled up on the first SMs the
+// linear freed).
 template <int HD, int KVQ>
 __global__ void rope_kv_kernel(uint16_t* __restrict__ qkv, int B, int S, int row_stride, int H, fp_kv_view kv,
                                const int32_t* __restrict__ pos, const float* __restrict__ cs, int32_t* err) {
-  pdl_trigger();
   pdl_wait();
   constexpr int E = HD / 32;
   const int Hkv = kv.n_kv_heads;

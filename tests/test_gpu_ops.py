@@ -175,7 +175,9 @@ def test_linear_residual_in_place(fp):
 
 
 # ---------------------------------------------------------------- rows
-@pytest.mark.parametrize("m,d,stride,offset", [(1, 512, 1, 0), (7, 4096, 1, 0), (3, 1024, 5, 4)])
+# rows from a ragged single warp's worth (d 40) to 40960 elements
+@pytest.mark.parametrize("m,d,stride,offset", [(1, 512, 1, 0), (7, 4096, 1, 0), (3, 1024, 5, 4), (32, 8192, 1, 0),
+                                              (2, 8200, 1, 0), (2, 24576, 2, 1), (3, 40, 1, 0), (1, 40960, 1, 0)])
 def test_rmsnorm(fp, m, d, stride, offset):
     rows = m * stride
     x = synth.uniform_bf16(21, d, (rows, d), -3, 3)
