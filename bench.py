@@ -110,8 +110,8 @@ NCU_TRAFFIC = {
     ("l70b", "lin_qkv"): {"bytes": 45146368, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
     ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
     ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "bd39d79e47b0ba01"},
-    ("l70b", "attn"): {"bytes": 149525504, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
-    ("l7b", "attn"): {"bytes": 81390848, "units": 8 * 612, "src": "fp_attention.cu", "sha": "e9d5e1e341aa3334"},
+    ("l70b", "attn"): {"bytes": 149513984, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "cc8ece47f7be26c7"},
+    ("l7b", "attn"): {"bytes": 81405952, "units": 8 * 612, "src": "fp_attention.cu", "sha": "cc8ece47f7be26c7"},
     ("l7b", "lm_head"): {"bytes": 270125824, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
     ("l7b", "lin_gu"): {"bytes": 94427904, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
     ("l7b", "lin_qkv"): {"bytes": 50466304, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
