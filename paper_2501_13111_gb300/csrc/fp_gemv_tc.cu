@@ -1,5 +1,5 @@
-// Decode linear for int4 group-128 weights at 17-64 tokens on the tcgen05
-// tensor cores.
+// Decode linear for int4 group-128 (and int8 per-channel) weights at 17-64
+// tokens on the tcgen05 tensor cores.
 //
 // y[m][n] = sum_k x[m][k] (q[n][k] - z[n][g]) s[n][g], g = k / 128, the
 // weight-only linear of a decoder block (QKV, O, gate+up, down) while the
@@ -38,6 +38,11 @@
 // last CTA to finish that slice (a ticket per slice) sums them in CTA order
 // and runs the epilogue -- residual add, SwiGLU, bf16 or fp32 store.
 //
+// int8 per-channel weights, y[m][n] = s[n] sum_k x[m][k] q[n][k], take the
+// same pipeline with items of 128 k (64 k of each matrix with SwiGLU): the
+// codes are widened exactly to bf16 (the integer q) and the row scale
+// multiplies the fp32 sums in the epilogue.
+//
 // Every mbarrier wait is bounded; past the limit the thread records error 2
 // in the error word, the CTA stops and releases TMEM after its copies and
 // MMAs have completed.
@@ -57,23 +62,26 @@ constexpr uint32_t kQ4TmemCols = 512;
 constexpr int kQ4Rows = 128;
 constexpr int kQ4MinSmem = 116 * 1024;  // above half an SM: one CTA (and one TMEM owner) per SM
 
-// An item is GPI consecutive 128-k groups of one row tile (of the gate and
-// the up tile with SwiGLU).  Without SwiGLU two groups per item (K a multiple
-// of 256) halve the hand-offs per byte: each item then carries 16 KB of
-// codes, as a SwiGLU item does.
-template <int MT, int NR, int GPI>
+// An item is KI consecutive k of one row tile (of the gate and the up tile
+// with SwiGLU), 8 or 16 KB of codes: int4 one 128-k group, or two where K is
+// a multiple of 256 and there is no SwiGLU; int8 128 k, or 64 k of each
+// matrix with SwiGLU.  Larger items halve the hand-offs per byte.
+template <int MT, int NR, int WQ, int KI>
 struct Q4Geom {
-  static_assert(GPI == 1 || NR == 1, "SwiGLU items hold one group of each matrix");
-  // each thread takes every other item: a whole group of its row (SwiGLU: of
-  // the gate or the up row; GPI 2: the first or the second group), otherwise
-  // half of one
-  static constexpr int kChunks = (NR == 2 || GPI == 2) ? 4 : 2;  // 16-byte code chunks per thread and item
+  static_assert(WQ == FP_W_INT8 || KI % 128 == 0, "int4 items hold whole groups");
+  static constexpr int kRowBytes = WQ == FP_W_INT8 ? KI : KI / 2;  // codes of one row of an item
+  // each thread takes every other item: its row's codes of the item (SwiGLU:
+  // of the gate or the up row), otherwise half of them
+  static constexpr int kThreadBytes = NR == 2 ? kRowBytes : kRowBytes / 2;
+  static constexpr int kChunks = kThreadBytes / 16;     // 16-byte code chunks per thread and item
+  static_assert(kChunks == 2 || kChunks == 4, "two or four chunks per thread");
+  static_assert(WQ == FP_W_INT4_G128 || kChunks == 4, "int8: one 32-column TMEM store per thread and item");
   static constexpr int kCodeBytes = kQ4DeqWarps * 32 * kChunks * 16;  // one ring stage, all threads
-  static constexpr int kXBytes = GPI * MT * 256;         // x [MT][128 GPI] bf16 as [MT][64] boxes
+  static constexpr int kXBytes = MT * KI * 2;            // x [MT][KI] bf16 as [MT][64] boxes
   // independent accumulation chains per matrix
   static constexpr int kChains = MT == 64 ? 2 / NR : 4 / NR;
   static constexpr int kDCols = NR * kChains * MT;       // fp32 accumulators
-  static constexpr int kACols = NR * GPI * 64;           // the item's bf16 pairs
+  static constexpr int kACols = NR * KI / 2;             // the item's bf16 pairs
   static constexpr int kASlots = std::min(6, ((int)kQ4TmemCols - kDCols) / kACols);
   // x stage a travels with A slot a: one barrier per item says both are ready
   // and one commit frees both
@@ -134,16 +142,31 @@ FP_DEV void deq_word(uint32_t w, uint32_t zz, uint32_t ss, uint32_t* out) {
   }
 }
 
+// One word of four int8 codes -> two bf16 pairs q (exact).  Byte b of
+// w ^ 0x80808080 is q_b + 128; placed under the exponent of 2^23 it gives the
+// float 2^23 + q_b + 128, from which one subtraction leaves q_b exactly, and
+// an integer of magnitude <= 127 is exact in bf16: the float's upper half.
+FP_DEV void i8_word(uint32_t w, uint32_t* out) {
+  const uint32_t u = w ^ 0x80808080u;
+  float f[4];
+#pragma unroll
+  for (int b = 0; b < 4; ++b) f[b] = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7440 + b)) - 8388736.0f;
+  out[0] = __byte_perm(__float_as_uint(f[0]), __float_as_uint(f[1]), 0x7632);
+  out[1] = __byte_perm(__float_as_uint(f[2]), __float_as_uint(f[3]), 0x7632);
+}
+
 FP_DEV long long q4_cta_of(long long i, long long C, long long total) { return ((i + 1) * C - 1) / total; }
 
-template <int MT, int EPI, int GPI>
+template <int MT, int EPI, int WQ, int KI>
 __global__ void __launch_bounds__(kQ4Threads, 1)
     gemv_q4tc_kernel(const __grid_constant__ CUtensorMap map_x, const uint8_t* __restrict__ codes, int M, int N,
                      const uint16_t* __restrict__ scales, const uint16_t* __restrict__ zeros, const uint16_t* R,
                      void* Y, long long total, int S, int V, float* __restrict__ ws, unsigned* __restrict__ counters,
                      int32_t* err) {
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
-  using G = Q4Geom<MT, NR, GPI>;
+  using G = Q4Geom<MT, NR, WQ, KI>;
+  constexpr bool I4 = WQ == FP_W_INT4_G128;
+  constexpr int GPI = I4 ? KI / 128 : 1;  // int4: groups per item
   constexpr int CS = kQ4CodeStages, XS = G::kXStages, NA = G::kASlots, MQ = MT / 4, DW = kQ4DeqWarps;
   constexpr int NCH = G::kChains, CK = G::kChunks;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -160,7 +183,7 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
   const long long C = gridDim.x, c = blockIdx.x;
   const long long begin = c * total / C, end = (c + 1) * total / C;
   const int L = (int)(end - begin);
-  const int SI = S / GPI;  // items per row tile
+  const int SI = S * 128 / KI;  // items per row tile (S: 128-k groups per row)
   auto fail = [&]() {
     *abort_flag = 1;
     if (err) atomicExch(err, 2);
@@ -206,7 +229,7 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
         uint8_t* xs = x_ring + s * G::kXBytes;
         mbar_expect_tx(&afull[s], G::kXBytes);
 #pragma unroll
-        for (int bx = 0; bx < 2 * GPI; ++bx) tma_load_2d(xs + bx * MT * 128, &map_x, g * GPI * 128 + bx * 64, 0, &afull[s]);
+        for (int bx = 0; bx < KI / 64; ++bx) tma_load_2d(xs + bx * MT * 128, &map_x, g * KI + bx * 64, 0, &afull[s]);
         issued = q + 1;
       }
       // copies still in flight land before the CTA leaves (their stages are its
@@ -235,12 +258,12 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
         // MMAs of one issuer never share an accumulator, and the two issuers'
         // chains are disjoint
 #pragma unroll
-        for (int kk = 0; kk < 8 * GPI; ++kk) {
+        for (int kk = 0; kk < KI / 16; ++kk) {
           const int r = NR == 2 ? mw : 0;
           if (NR == 1 && (kk & 1) != mw) continue;
           // descriptor start addresses count 16-byte units; k-step kk reads A
           // columns 8 kk .. +7 (of matrix r) and x box kk / 4
-          tc_mma_ts(tmem + (r * NCH + kk % NCH) * MT, ta + r * 64 + kk * 8,
+          tc_mma_ts(tmem + (r * NCH + kk % NCH) * MT, ta + r * (KI / 2) + kk * 8,
                     xd + (uint64_t)(((kk >> 2) * MT * 128 + (kk & 3) * 32) >> 4), idesc, (first && kk < NCH) ? 0u : 1u);
         }
         tc_commit(&aempty[a]);  // A slot a and x stage a have been read
@@ -264,11 +287,11 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
     const int qd = warp & 3, team = warp >> 3, half = (warp >> 2) & 1, lr = qd * 32 + lane;
     const int pt = warp >> 2;  // epilogue: tokens [pt MQ, (pt + 1) MQ)
     const int rm = NR == 2 ? half : 0;
-    const int gsel = GPI == 2 ? half : 0;                    // this warp's group of the item
-    const int cbase = (NR == 1 && GPI == 1) ? 2 * half : 0;  // first 16-byte chunk of the group's 64 bytes
-    const int acol = NR == 2 ? rm * 64 : GPI == 2 ? half * 64 : half * 32;
+    const int gsel = (I4 && GPI == 2) ? half : 0;                   // int4: this warp's group of the item
+    const int tboff = NR == 1 ? half * G::kThreadBytes : 0;         // this warp's bytes of the item's row
+    const int acol = NR == 2 ? rm * (KI / 2) : half * (KI / 4);
     const uint32_t lane_base = tmem + ((uint32_t)(qd * 32) << 16);
-    const long long row_bytes = (long long)S * 64;
+    const long long row_bytes = (long long)SI * G::kRowBytes;
 
     // ---- this thread's code ring: its n-th own item (team + 2 n) in stage
     // n % CS, chunk i at [stage][i][thread] (a warp's loads of one chunk are
@@ -279,14 +302,14 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
     const uint8_t* src = nullptr;
     auto set_src = [&]() {
       const long long rr = min(ib * kQ4Rows + lr, Nout - 1) + rm * Nout;
-      src = codes + rr * row_bytes + gsel * 64 + cbase * 16;
+      src = codes + rr * row_bytes + tboff;
     };
     if (own > 0) set_src();
     auto issue = [&](int n) {  // called for n = 0, 1, 2, ... in order
       if (n < own) {
         uint8_t* d = my_ring + (size_t)(n % CS) * G::kCodeBytes;
 #pragma unroll
-        for (int i = 0; i < CK; ++i) q4_cp16(d + i * (DW * 32 * 16), src + (long long)ig * (GPI * 64) + i * 16);
+        for (int i = 0; i < CK; ++i) q4_cp16(d + i * (DW * 32 * 16), src + (long long)ig * G::kRowBytes + i * 16);
         ig += 2;
         if (ig >= SI) {
           while (ig >= SI) ig -= SI, ++ib;
@@ -299,14 +322,17 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
 #pragma unroll 1
     for (int n = 0; n < CS - 1; ++n) issue(n);
 
-    // scales and zeros of the row, V groups (VI items) per load, one chunk
-    // ahead (S % V == 0, so a chunk never crosses a row tile)
-    const int VI = V / GPI;
-    uint4 s_cur, z_cur, s_nxt = make_uint4(0u, 0u, 0u, 0u), z_nxt = s_nxt;
+    // int4: scales and zeros of the row, V groups (VI items) per load, one
+    // chunk ahead (S % V == 0, so a chunk never crosses a row tile); int8 has
+    // one scale per row, applied in the epilogue
+    const int VI = I4 ? V / GPI : 1;
+    uint4 s_cur = make_uint4(0u, 0u, 0u, 0u), z_cur = s_cur, s_nxt = s_cur, z_nxt = s_cur;
     auto load_chunk = [&](int bb, int g0, uint4& sv, uint4& zv) {  // g0: first item of the chunk
-      const long long idx = (long long)(min(bb * kQ4Rows + lr, Nout - 1) + rm * Nout) * S + (long long)g0 * GPI;
-      sv = ld_groups(scales + idx, V);
-      zv = ld_groups(zeros + idx, V);
+      if constexpr (I4) {
+        const long long idx = (long long)(min(bb * kQ4Rows + lr, Nout - 1) + rm * Nout) * S + (long long)g0 * GPI;
+        sv = ld_groups(scales + idx, V);
+        zv = ld_groups(zeros + idx, V);
+      }
     };
     // (row tile, item) of the current item and its place j in the chunk of VI
     // items, advanced without divisions
@@ -340,29 +366,42 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
           wv[i] = *reinterpret_cast<const uint4*>(my_ring + (size_t)(n % CS) * G::kCodeBytes + i * (DW * 32 * 16));
         issue(n + CS - 1);  // refills the stage read one own item ago
 
-        const uint32_t sb = bf16_at(s_cur, j * GPI + gsel);
-        const uint32_t zb = f2bf(128.f + bf2f((uint16_t)bf16_at(z_cur, j * GPI + gsel)));
-        const uint32_t ss = sb | (sb << 16), zz = zb | (zb << 16);
         const uint32_t ta = lane_base + G::kDCols + a * G::kACols + acol;
         bool ok = true;
+        auto slot_free = [&]() {  // the first columns are converted while the slot drains
+          ok = mbar_wait_sleep(&aempty[a], ((q / NA) & 1) ^ 1);
+          ok = __all_sync(0xffffffffu, ok) && !__any_sync(0xffffffffu, *abort_flag != 0);
+          if (ok) tc_fence_after();
+          return ok;
+        };
+        if constexpr (I4) {
+          const uint32_t sb = bf16_at(s_cur, j * GPI + gsel);
+          const uint32_t zb = f2bf(128.f + bf2f((uint16_t)bf16_at(z_cur, j * GPI + gsel)));
+          const uint32_t ss = sb | (sb << 16), zz = zb | (zb << 16);
 #pragma unroll
-        for (int h2 = 0; h2 < CK / 2; ++h2) {  // 32 columns (two chunks) per store
-          uint32_t av[32];
+          for (int h2 = 0; h2 < CK / 2; ++h2) {  // 32 columns (two chunks) per store
+            uint32_t av[32];
 #pragma unroll
-          for (int i = 0; i < 2; ++i) {
-            const uint4 w = wv[2 * h2 + i];
-            deq_word(w.x, zz, ss, av + i * 16);
-            deq_word(w.y, zz, ss, av + i * 16 + 4);
-            deq_word(w.z, zz, ss, av + i * 16 + 8);
-            deq_word(w.w, zz, ss, av + i * 16 + 12);
+            for (int i = 0; i < 2; ++i) {
+              const uint4 w = wv[2 * h2 + i];
+              deq_word(w.x, zz, ss, av + i * 16);
+              deq_word(w.y, zz, ss, av + i * 16 + 4);
+              deq_word(w.z, zz, ss, av + i * 16 + 8);
+              deq_word(w.w, zz, ss, av + i * 16 + 12);
+            }
+            if (h2 == 0 && !slot_free()) break;
+            tc_st32(ta + h2 * 32, av);
           }
-          if (h2 == 0) {  // the first columns are converted while the slot drains
-            ok = mbar_wait_sleep(&aempty[a], ((q / NA) & 1) ^ 1);
-            ok = __all_sync(0xffffffffu, ok) && !__any_sync(0xffffffffu, *abort_flag != 0);
-            if (!ok) break;
-            tc_fence_after();
+        } else {
+          uint32_t av[32];  // four chunks of 16 codes: 32 columns of bf16 pairs
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            i8_word(wv[i].x, av + i * 8);
+            i8_word(wv[i].y, av + i * 8 + 2);
+            i8_word(wv[i].z, av + i * 8 + 4);
+            i8_word(wv[i].w, av + i * 8 + 6);
           }
-          tc_st32(ta + h2 * 32, av);
+          if (slot_free()) tc_st32(ta, av);
         }
         if (!ok) {
           if (lane == 0) fail();
@@ -401,12 +440,21 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
       ++seg;
 
       const int row = b * kQ4Rows + lr;
+      // int8: the row scales (gate and up rows with SwiGLU) multiply the sums
+      float sg = 1.f, su = 1.f;
+      if constexpr (!I4) {
+        const int rc = min(row, Nout - 1);
+        sg = bf2f(scales[rc]);
+        su = bf2f(scales[(NR - 1) * Nout + rc]);
+      }
       // r: the residual R[m][row], read before any store (R may be Y itself)
       auto resid = [&](int m) {
         return (EPI == FP_EPI_RESID && m < M && row < Nout) ? bf2f(R[(long long)m * Nout + row]) : 0.f;
       };
       auto finish = [&](int m, float v, float u, float r) {
         const long long o = (long long)m * Nout + row;
+        v *= sg;
+        u *= su;
         if constexpr (EPI == FP_EPI_STORE) ((uint16_t*)Y)[o] = f2bf(v);
         else if constexpr (EPI == FP_EPI_RESID) ((uint16_t*)Y)[o] = f2bf(r + v);
         else if constexpr (EPI == FP_EPI_SWIGLU) ((uint16_t*)Y)[o] = f2bf(silu(v) * u);
@@ -495,74 +543,92 @@ static int q4_mt(int M) { return M <= 32 ? 32 : 64; }
 static int q4_v(int groups) { return groups % 8 == 0 ? 8 : groups % 4 == 0 ? 4 : groups % 2 == 0 ? 2 : 1; }
 
 bool q4tc_ok(int wquant, int epi, int M, int N, int K) {
-  if (wquant != FP_W_INT4_G128 || M < 17 || M > 64 || N < 1 || K < 128 || K % 128 != 0) return false;
+  if ((wquant != FP_W_INT4_G128 && wquant != FP_W_INT8) || M < 17 || M > 64 || N < 1 || K < 128 || K % 128 != 0)
+    return false;
   if (epi == FP_EPI_SWIGLU && N % 2 != 0) return false;
   const long long nout = epi == FP_EPI_SWIGLU ? N / 2 : N;
   const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
   return blocks * kQ4DeqWarps <= kLinTicketSlots && tensor_maps_available();
 }
 
+// int4 always; int8 beyond 32 tokens or for long rows.  Measured at the
+// 70B-shaped block's linears, microseconds on tcgen05 against mma.sync: 32
+// tokens QKV 45.3 / 41.0, O 39.3 / 35.8, gate+up 173.9 / 165.4, down (K
+// 28672) 86.2 / 118.9; 64 tokens 48.8 / 81.3, 45.1 / 70.3, 180.3 / 267.1,
+// 96.0 / 204.7.  An int8 item carries half the weights of an int4 item for
+// the same hand-offs, while the mma.sync GEMV's cost grows with the tokens.
+bool q4tc_preferred(int wquant, int M, int K) { return wquant != FP_W_INT8 || M > 32 || K >= 16384; }
+
 size_t q4tc_ws_bytes(int epi, int M, int N, int K) {
   const int nr = epi == FP_EPI_SWIGLU ? 2 : 1;
   const long long nout = nr == 2 ? N / 2 : N;
   const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
-  const long long ctas = std::min<long long>(blocks * (K / 128), q4_sms());
+  const long long ctas = std::min<long long>(blocks * (K / 64), q4_sms());  // items are at least 64 k
   return (size_t)kLinTicketSlots * 4 + (size_t)(blocks + ctas) * M * nr * kQ4Rows * 4;
 }
 
-template <int MT, int EPI, int GPI>
+template <int MT, int EPI, int WQ, int KI>
 static cudaError_t launch_q4_t(const uint8_t* codes, const CUtensorMap& mx, int M, int N, int K,
                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* Y, void* ws,
                                int32_t* err, cudaStream_t s) {
   constexpr int NR = EPI == FP_EPI_SWIGLU ? 2 : 1;
-  auto kern = gemv_q4tc_kernel<MT, EPI, GPI>;
-  const int smem = std::max(Q4Geom<MT, NR, GPI>::kSmem, kQ4MinSmem);
+  auto kern = gemv_q4tc_kernel<MT, EPI, WQ, KI>;
+  const int smem = std::max(Q4Geom<MT, NR, WQ, KI>::kSmem, kQ4MinSmem);
   static std::atomic<unsigned long long> attr{0};
   FP_CUDA_TRY(smem_limit_once(kern, smem, &attr));
   const int nout = NR == 2 ? N / 2 : N;
   const long long blocks = (nout + kQ4Rows - 1) / kQ4Rows;
   const int S = K / 128;
-  const long long total = blocks * (S / GPI);  // items
+  const long long total = blocks * (K / KI);  // items
   const int ctas = (int)std::min<long long>(total, q4_sms());
   unsigned* counters = (unsigned*)ws;
   float* part = (float*)((char*)ws + (size_t)kLinTicketSlots * 4);
   return launch(kern, dim3(ctas), dim3(kQ4Threads), (size_t)smem, s, mx, codes, M, N, scales, zeros, R, Y, total, S,
-                q4_v(S), part, counters, err);
+                WQ == FP_W_INT4_G128 ? q4_v(S) : 1, part, counters, err);
 }
 
-template <int MT>
-static cudaError_t launch_q4_m(int epi, const uint8_t* mw, const CUtensorMap& mx, int M, int N, int K,
+// k per item: int4 two groups where K allows (SwiGLU items already carry two
+// matrices' groups), else one; int8 128, with SwiGLU 64 of each matrix
+template <int MT, int WQ>
+static cudaError_t launch_q4_w(int epi, const uint8_t* mw, const CUtensorMap& mx, int M, int N, int K,
                                const uint16_t* scales, const uint16_t* zeros, const uint16_t* R, void* Y, void* ws,
                                int32_t* err, cudaStream_t s) {
-  // two groups per item where K allows (SwiGLU items already carry two)
-  const bool two = (K / 128) % 2 == 0;
+  constexpr bool I4 = WQ == FP_W_INT4_G128;
+  constexpr int K2 = I4 ? 256 : 128;  // the larger item
+  const bool two = I4 && (K / 128) % 2 == 0;
   switch (epi) {
     case FP_EPI_STORE:
-      return two ? launch_q4_t<MT, FP_EPI_STORE, 2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
-                 : launch_q4_t<MT, FP_EPI_STORE, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+      return two ? launch_q4_t<MT, FP_EPI_STORE, WQ, K2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
+                 : launch_q4_t<MT, FP_EPI_STORE, WQ, 128>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
     case FP_EPI_RESID:
-      return two ? launch_q4_t<MT, FP_EPI_RESID, 2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
-                 : launch_q4_t<MT, FP_EPI_RESID, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
-    case FP_EPI_SWIGLU: return launch_q4_t<MT, FP_EPI_SWIGLU, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+      return two ? launch_q4_t<MT, FP_EPI_RESID, WQ, K2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
+                 : launch_q4_t<MT, FP_EPI_RESID, WQ, 128>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+    case FP_EPI_SWIGLU:
+      return launch_q4_t<MT, FP_EPI_SWIGLU, WQ, I4 ? 128 : 64>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
     default:
-      return two ? launch_q4_t<MT, FP_EPI_F32, 2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
-                 : launch_q4_t<MT, FP_EPI_F32, 1>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
+      return two ? launch_q4_t<MT, FP_EPI_F32, WQ, K2>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s)
+                 : launch_q4_t<MT, FP_EPI_F32, WQ, 128>(mw, mx, M, N, K, scales, zeros, R, Y, ws, err, s);
   }
 }
 
-cudaError_t launch_q4tc(int epi, const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
-                        const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
-                        int32_t* err, cudaStream_t s) {
-  if (!q4tc_ok(FP_W_INT4_G128, epi, M, N, K)) return cudaErrorInvalidValue;
+cudaError_t launch_q4tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
+                        const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y, void* ws,
+                        size_t ws_bytes, int32_t* err, cudaStream_t s) {
+  if (!q4tc_ok(wquant, epi, M, N, K)) return cudaErrorInvalidValue;
   if (!ws || ws_bytes < q4tc_ws_bytes(epi, M, N, K)) return cudaErrorInvalidValue;
   CUtensorMap mx;
   const int mt = q4_mt(M);
   const uint8_t* mw = (const uint8_t*)codes;
   // x [M][K] bf16, box [mt rows][64]
   if (!make_tensor_map(&mx, x, M, K, 2, mt, 64, 128)) return cudaErrorInvalidValue;
+  const bool i8 = wquant == FP_W_INT8;
   switch (mt) {
-    case 32: return launch_q4_m<32>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s);
-    default: return launch_q4_m<64>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s);
+    case 32:
+      return i8 ? launch_q4_w<32, FP_W_INT8>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s)
+                : launch_q4_w<32, FP_W_INT4_G128>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s);
+    default:
+      return i8 ? launch_q4_w<64, FP_W_INT8>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s)
+                : launch_q4_w<64, FP_W_INT4_G128>(epi, mw, mx, M, N, K, scales, zeros, residual, y, ws, err, s);
   }
 }
 

@@ -834,9 +834,11 @@ cudaError_t launch_linear(int wquant, int epi, const uint16_t* x, int M, int N, 
   if (btc_ok(wquant, epi, M, N, K) && btc_preferred(epi, N, K) && ((uintptr_t)x & 15) == 0 &&
       ((uintptr_t)codes & 15) == 0)
     return launch_btc(epi, x, M, N, K, codes, residual, y, ws, ws_bytes, err, s);
-  // int4 at 9-64 tokens: the tensor-core path (TMA needs 16-byte aligned x and codes)
-  if (q4tc_ok(wquant, epi, M, N, K) && ((uintptr_t)x & 15) == 0 && ((uintptr_t)codes & 15) == 0)
-    return launch_q4tc(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, err, s);
+  // int4 and int8 at 17-64 tokens: the tensor-core path, weights expanded into
+  // TMEM (TMA needs 16-byte aligned x and codes)
+  if (q4tc_ok(wquant, epi, M, N, K) && q4tc_preferred(wquant, M, K) && ((uintptr_t)x & 15) == 0 &&
+      ((uintptr_t)codes & 15) == 0)
+    return launch_q4tc(wquant, epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, err, s);
   if (mma_ok(wquant, M, N, K)) {
     switch (wquant) {
       case FP_W_BF16: return launch_mma<FP_W_BF16>(epi, x, M, N, K, codes, scales, zeros, residual, y, ws, ws_bytes, s, err);

@@ -73,12 +73,13 @@ cudaError_t launch_linear_gptq4(int epi, const uint16_t* x, int M, int N, int K,
                                 const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
                                 cudaStream_t s, int32_t* err);
 
-// ---- int4 decode linear at 9-64 tokens on tcgen05 (fp_gemv_tc.cu)
+// ---- int4 / int8 decode linear at 17-64 tokens on tcgen05 (fp_gemv_tc.cu)
 bool q4tc_ok(int wquant, int epi, int M, int N, int K);
+bool q4tc_preferred(int wquant, int M, int K);
 size_t q4tc_ws_bytes(int epi, int M, int N, int K);
-cudaError_t launch_q4tc(int epi, const uint16_t* x, int M, int N, int K, const void* codes, const uint16_t* scales,
-                        const uint16_t* zeros, const uint16_t* residual, void* y, void* ws, size_t ws_bytes,
-                        int32_t* err, cudaStream_t s);
+cudaError_t launch_q4tc(int wquant, int epi, const uint16_t* x, int M, int N, int K, const void* codes,
+                        const uint16_t* scales, const uint16_t* zeros, const uint16_t* residual, void* y, void* ws,
+                        size_t ws_bytes, int32_t* err, cudaStream_t s);
 
 // ---- bf16 decode linear at 17-64 tokens on tcgen05, TMA-fed (fp_gemv_btc.cu)
 bool btc_ok(int wquant, int epi, int M, int N, int K);

@@ -211,6 +211,11 @@ for tag, (wq, d, H, Hkv, f, Mdec) in {"7b": (1, 4096, 32, 32, 11008, 8), "13b": 
     CASES[f"{tag}-down"] = ("linear", (wq, 1, Mdec, d, f))
     CASES[f"{tag}-lmhead"] = ("linear", (0, 3, Mdec, 32000, d))
     CASES[f"{tag}-argmax"] = ("argmax", (Mdec, 32000))
+# the 70B-shaped block's linears with int8 weights at the 70B decode batch
+for _tag, (_epi, _n, _k) in {"qkv": (0, 10240, 8192), "o": (1, 8192, 8192), "gu": (2, 57344, 8192),
+                             "down": (1, 8192, 28672)}.items():
+    CASES[f"70b-i8-{_tag}"] = ("linear", (1, _epi, 32, _n, _k))
+    CASES[f"70b-i8-{_tag}-b64"] = ("linear", (1, _epi, 64, _n, _k))
 CASES["7b-attn"] = ("attention", (8, 32, 32, 128, 612, 0))
 CASES["13b-attn"] = ("attention", (16, 40, 40, 128, 1124, 0))
 CASES["70b-attn"] = ("attention", (32, 64, 8, 128, 2148, 1))

@@ -159,6 +159,46 @@ def test_linear_int4_tensor_core(fp, m, n, k, epi):
         assert rel_err(got, y) <= tol, (m, n, k, epi, tol, rel_err(got, y))
 
 
+@pytest.mark.parametrize("m,n,k,epi", [
+    (17, 300, 4096, 1), (32, 1000, 8192, 0), (33, 256, 1152, 3), (48, 520, 2048, 2), (64, 136, 11008, 1),
+    (32, 2048, 3584, 3), (17, 1152, 1152, 0), (64, 2000, 128, 2), (40, 16384, 256, 0), (20, 384, 1088, 0),
+    (24, 256, 16384, 1), (32, 512, 16384, 2), (17, 300, 20480, 3)])
+def test_linear_int8_tensor_core(fp, m, n, k, epi):
+    """int8 per-channel weights at 17-64 tokens: beyond 32 tokens, or with K
+    of 16384 or more, the codes widened exactly to bf16 in TMEM, products
+    accumulated in fp32 on tcgen05, the row scale applied to the sums; else
+    the mma.sync GEMV.  Cases: ragged row tiles, tokens padded to 32 / 64,
+    SwiGLU items of 64 k (K 128: two per row), row tiles shared by several
+    CTAs and CTAs covering whole tiles; K = 1088 (not a multiple of 128)
+    always takes the mma.sync GEMV."""
+    w = synth.weight_bf16(60 + m, 0, 1, (n, k))
+    x = synth.uniform_bf16(61, m, (m, k), -2.0, 2.0)
+    r = synth.uniform_bf16(62, m, (m, n), -1.0, 1.0)
+    codes, scales, zeros = _quantized_on_device(fp, 1, w)
+    _, wd = quant.quantize_weight(w, 1)
+    xf = quant.bf16_to_f32(x).astype(np.float64)
+    nout = n // 2 if epi == 2 else n
+    out = empty(m * nout * (4 if epi == 3 else 2))
+    ws_b = fp.fp_op_linear_workspace_bytes(1, m, n, k)
+    ws = empty(max(ws_b, 16))
+    fp.fp_op_linear(1, epi, ptr(dev(x)), m, n, k, ptr(codes), ptr(scales), ptr(zeros), ptr(dev(r)), ptr(out),
+                    ptr(ws), ws_b)
+    if epi == 3:
+        got = host(out, np.float32).reshape(m, n).astype(np.float64)
+    else:
+        got = quant.bf16_to_f32(host(out, np.uint16)).reshape(m, nout).astype(np.float64)
+    y = xf @ wd.T
+    if epi == 1:
+        y = quant.bf16_to_f32(r).astype(np.float64) + y
+    elif epi == 2:
+        y = M.silu(y[:, :nout]) * y[:, nout:]
+    # the tensor-core path sees x and the codes exactly (the mma.sync GEMV
+    # stages x in fp16): fp32 sums against the exact product
+    tight = k % 128 == 0 and (m > 32 or k >= 16384)
+    tol = (1e-4 if epi == 3 else 6e-3) if tight else TAU[1] / 4
+    assert rel_err(got, y) <= tol, (m, n, k, epi, tol, rel_err(got, y))
+
+
 def test_linear_residual_in_place(fp):
     m, n, k = 5, 64, 256
     w = synth.weight_bf16(3, 0, 1, (n, k))
