@@ -105,10 +105,10 @@ def class_roofline(cls, kb, cls_time, launches, peak):
 # bench's B x context.
 NCU_TRAFFIC = {
     # profiles/dram_traffic_l70b.md and dram_traffic_l7b.md: microbench cases, one launch each
-    ("l70b", "lin_gu"): {"bytes": 273308928, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
-    ("l70b", "lin_down"): {"bytes": 130883584, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
-    ("l70b", "lin_qkv"): {"bytes": 45146368, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
-    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "1f728c8c1b2204e6"},
+    ("l70b", "lin_gu"): {"bytes": 273285632, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
+    ("l70b", "lin_down"): {"bytes": 130825472, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
+    ("l70b", "lin_qkv"): {"bytes": 45146624, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
+    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
     ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "bd39d79e47b0ba01"},
     ("l70b", "attn"): {"bytes": 149513984, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "cc8ece47f7be26c7"},
     ("l7b", "attn"): {"bytes": 81405952, "units": 8 * 612, "src": "fp_attention.cu", "sha": "cc8ece47f7be26c7"},
