@@ -99,37 +99,51 @@ def class_roofline(cls, kb, cls_time, launches, peak):
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of the
 # decode kernels from the ncu captures summarised in profiles/ (microbench
 # cases of the workload's shapes), keyed by (workload, kernel class), with the
-# sha256 prefix of the kernel's source at capture time: a changed source makes
-# the figure stale and it is reported as null.  Attention traffic is per
+# sha256 prefix of the kernel's source code at capture time (comments and
+# blank lines left out, see source_code_sha): changed code makes the figure
+# stale and it is reported as null.  Attention traffic is per
 # cached token row (units = B x context of the capture) and scales with the
 # bench's B x context.
 NCU_TRAFFIC = {
     # profiles/dram_traffic_l70b.md and dram_traffic_l7b.md: microbench cases, one launch each
-    ("l70b", "lin_gu"): {"bytes": 273285632, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
-    ("l70b", "lin_down"): {"bytes": 130825472, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
-    ("l70b", "lin_qkv"): {"bytes": 45146624, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
-    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "121d655c01445061"},
-    ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "bd39d79e47b0ba01"},
-    ("l70b", "attn"): {"bytes": 149513984, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "cc8ece47f7be26c7"},
-    ("l7b", "attn"): {"bytes": 81405952, "units": 8 * 612, "src": "fp_attention.cu", "sha": "cc8ece47f7be26c7"},
-    ("l7b", "lm_head"): {"bytes": 270125824, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
-    ("l7b", "lin_gu"): {"bytes": 94427904, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
-    ("l7b", "lin_qkv"): {"bytes": 50466304, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
-    ("l7b", "lin_o"): {"bytes": 16945920, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
-    ("l7b", "lin_down"): {"bytes": 45368576, "units": None, "src": "fp_linear.cu", "sha": "131cc1c359c0a3ad"},
+    ("l70b", "lin_gu"): {"bytes": 273285632, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
+    ("l70b", "lin_down"): {"bytes": 130825472, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
+    ("l70b", "lin_qkv"): {"bytes": 45146624, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
+    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
+    ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "ac6ffae462038acd"},
+    ("l70b", "attn"): {"bytes": 149513984, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "011e2b422a5fa35c"},
+    ("l7b", "attn"): {"bytes": 81405952, "units": 8 * 612, "src": "fp_attention.cu", "sha": "011e2b422a5fa35c"},
+    ("l7b", "lm_head"): {"bytes": 270125824, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
+    ("l7b", "lin_gu"): {"bytes": 94427904, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
+    ("l7b", "lin_qkv"): {"bytes": 50466304, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
+    ("l7b", "lin_o"): {"bytes": 16945920, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
+    ("l7b", "lin_down"): {"bytes": 45368576, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
 }
+
+
+def source_code_sha(path):
+    """sha256 prefix of a C++/CUDA source with its comments, leading and
+    trailing blanks and empty lines left out: an edit of the comments keeps
+    it, any change of the code changes it."""
+    import hashlib
+    import re
+
+    with open(path, encoding="utf-8") as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", "", text)
+    lines = [line.strip() for line in text.splitlines()]
+    return hashlib.sha256("\n".join(line for line in lines if line).encode()).hexdigest()[:16]
 
 
 def ncu_traffic(cls, cfg_name, B, ctx):
     """Per-launch DRAM bytes of kernel class `cls` from the recorded capture, or None."""
-    import hashlib
-
     t = NCU_TRAFFIC.get((cfg_name, cls))
     if t is None:
         return None
     src = os.path.join(ROOT, "paper_2501_13111_gb300", "csrc", t["src"])
     try:
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        sha = source_code_sha(src)
     except OSError:
         return None
     if sha != t["sha"]:

@@ -9,24 +9,25 @@
 // lane each) and the tokens the N dimension of tcgen05.mma (M 128, N =
 // tokens rounded up to 32 or 64, K 16):
 //   warps 0-15  dequantise, in two teams of eight that take alternate
-//               items (two consecutive 128-k groups where K allows, else one;
-//               SwiGLU: one group of the gate and of the up tile): warp w
-//               owns TMEM lanes 32 (w % 4) .. +31 (one weight row per thread)
-//               and one group of the item (else half of it).  Each thread streams its
-//               own codes through a private cp.async ring in shared memory
-//               (no cross-warp handshake),
+//               items (KI consecutive k of a row tile; SwiGLU: of the gate
+//               and of the up tile): warp w owns TMEM lanes 32 (w % 4) .. +31
+//               (one weight row per thread) and the first or second half of
+//               the item's k (SwiGLU: the gate or the up row).  Each thread
+//               streams its own codes through a private cp.async ring in
+//               shared memory (no cross-warp handshake),
 //               forms bf16((q - z) s) -- exactly the prefill expansion --
 //               and stores them into an A slot of TMEM (tcgen05.st, two K
 //               elements per 32-bit column); afull / aempty hand the slots
 //               to the MMA thread and back;
-//   warp 16     TMA producer of x ([N][128] bf16 per group as two
+//   warp 16     TMA producer of x ([N][KI] bf16 per item as [N][64]
 //               128-byte-swizzled boxes, rows past M zero-filled) into a ring
 //               whose stage a goes with A slot a: afull[a] completes when the
 //               team's warps have stored the slot and the x bytes have
 //               landed, and one commit of the MMAs frees both (aempty[a]), so
 //               the MMA thread waits once and commits once per item;
-//   warp 17     allocates 512 TMEM columns and issues the MMAs (A from TMEM,
-//               B = x from shared memory) into fp32 TMEM accumulators.
+//   warps 17-18 issue the MMAs (A from TMEM, B = x from shared memory) into
+//               fp32 TMEM accumulators, each its own chains (SwiGLU: one
+//               matrix each); warp 17 also allocates the 512 TMEM columns.
 // MMAs (M 128, N <= 64, K 16) into one accumulator follow each other at
 // about 50 cycles, far above their math (N / 2 cycles), while MMAs into
 // different accumulators overlap: the k-steps of each matrix are spread
@@ -54,7 +55,7 @@
 
 namespace fpk {
 
-constexpr int kQ4CodeStages = 4;  // per-thread cp.async ring depth, one (own) group per stage
+constexpr int kQ4CodeStages = 4;  // per-thread cp.async ring depth, one (own) item per stage
 constexpr int kQ4DeqWarps = 16;
 constexpr int kQ4MmaWarps = 2;  // MMA issuers, each with its own accumulators
 constexpr int kQ4Threads = (kQ4DeqWarps + 1 + kQ4MmaWarps) * 32;
@@ -192,8 +193,8 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
   pdl_trigger();
   if (threadIdx.x == 0) {
     for (int a = 0; a < NA; ++a) {
-      // the eight warps of the group's team stored its A columns, and the x
-      // producer's expect_tx, completed by the bytes of the group's x
+      // the eight warps of the item's team stored its A columns, and the x
+      // producer's expect_tx, completed by the bytes of the item's x
       mbar_init(&afull[a], DW / 2 + 1);
       mbar_init(&aempty[a], kQ4MmaWarps);  // tcgen05.commit of the MMAs that read slot and stage
     }
@@ -281,9 +282,9 @@ __global__ void __launch_bounds__(kQ4Threads, 1)
     // ---------------- dequantise (+ epilogue)
     // two teams of eight warps take alternate items, so one team computes
     // while the other waits; within a team warp w owns TMEM lanes
-    // 32 (w % 4) .. +31 and, SwiGLU, the gate or the up rows, with two groups
-    // per item the first or the second group, otherwise the first or second
-    // half of the group
+    // 32 (w % 4) .. +31 and, SwiGLU, the gate or the up rows, otherwise the
+    // first or second half of the item's k (int4 with two groups per item:
+    // the first or the second group)
     const int qd = warp & 3, team = warp >> 3, half = (warp >> 2) & 1, lr = qd * 32 + lane;
     const int pt = warp >> 2;  // epilogue: tokens [pt MQ, (pt + 1) MQ)
     const int rm = NR == 2 ? half : 0;

@@ -58,6 +58,30 @@ def test_kernel_bytes_closed_forms():
     assert kb["attn"] == pytest.approx(B * S * a["n_kv_heads"] * a["head_dim"] * 2 * 2, rel=0.02)
 
 
+def test_source_code_sha_ignores_comments_only(tmp_path):
+    """The recorded ncu traffic stays valid across comment edits of a kernel's
+    source and goes stale on any code edit."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    base = "// header\n__global__ void k(int* p) {\n  p[0] = 1;  // store\n}\n"
+    variants = {
+        "same": base,
+        "comments": "/* block\n comment */\n// other header\n__global__ void k(int* p) {\n\n  p[0] = 1;\n}\n",
+        "code": "// header\n__global__ void k(int* p) {\n  p[0] = 2;  // store\n}\n",
+    }
+    sha = {}
+    for name, text in variants.items():
+        f = tmp_path / (name + ".cu")
+        f.write_text(text)
+        sha[name] = bench.source_code_sha(str(f))
+    assert sha["same"] == sha["comments"]
+    assert sha["same"] != sha["code"]
+    # every table entry names a source that exists
+    for (cfg, cls), t in bench.NCU_TRAFFIC.items():
+        assert os.path.exists(os.path.join(ROOT, "paper_2501_13111_gb300", "csrc", t["src"])), (cfg, cls)
+
+
 FAKE_SMI = """#!/bin/bash
 # stands in for nvidia-smi: refuses sampling periods below MIN_MS, else prints
 # one CSV sample per period (SM MHz counting up from 2000) until killed
