@@ -113,11 +113,11 @@ NCU_TRAFFIC = {
     ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "ac6ffae462038acd"},
     ("l70b", "attn"): {"bytes": 149513984, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "011e2b422a5fa35c"},
     ("l7b", "attn"): {"bytes": 81405952, "units": 8 * 612, "src": "fp_attention.cu", "sha": "011e2b422a5fa35c"},
-    ("l7b", "lm_head"): {"bytes": 270125824, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
-    ("l7b", "lin_gu"): {"bytes": 94427904, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
-    ("l7b", "lin_qkv"): {"bytes": 50466304, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
-    ("l7b", "lin_o"): {"bytes": 16945920, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
-    ("l7b", "lin_down"): {"bytes": 45368576, "units": None, "src": "fp_linear.cu", "sha": "3a9cd2f29f7f4695"},
+    ("l7b", "lm_head"): {"bytes": 270177792, "units": None, "src": "fp_linear.cu", "sha": "136661144db50e97"},
+    ("l7b", "lin_gu"): {"bytes": 94035456, "units": None, "src": "fp_linear.cu", "sha": "136661144db50e97"},
+    ("l7b", "lin_qkv"): {"bytes": 50459904, "units": None, "src": "fp_linear.cu", "sha": "136661144db50e97"},
+    ("l7b", "lin_o"): {"bytes": 16946176, "units": None, "src": "fp_linear.cu", "sha": "136661144db50e97"},
+    ("l7b", "lin_down"): {"bytes": 45368320, "units": None, "src": "fp_linear.cu", "sha": "136661144db50e97"},
 }
 
 
