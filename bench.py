@@ -106,10 +106,10 @@ def class_roofline(cls, kb, cls_time, launches, peak):
 # bench's B x context.
 NCU_TRAFFIC = {
     # profiles/dram_traffic_l70b.md and dram_traffic_l7b.md: microbench cases, one launch each
-    ("l70b", "lin_gu"): {"bytes": 273285632, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
-    ("l70b", "lin_down"): {"bytes": 130825472, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
-    ("l70b", "lin_qkv"): {"bytes": 45146624, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
-    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "b8a7b0a3d674ebb4"},
+    ("l70b", "lin_gu"): {"bytes": 273504512, "units": None, "src": "fp_gemv_tc.cu", "sha": "4ce5acf290c2928d"},
+    ("l70b", "lin_down"): {"bytes": 130917632, "units": None, "src": "fp_gemv_tc.cu", "sha": "4ce5acf290c2928d"},
+    ("l70b", "lin_qkv"): {"bytes": 45146880, "units": None, "src": "fp_gemv_tc.cu", "sha": "4ce5acf290c2928d"},
+    ("l70b", "lin_o"): {"bytes": 36759552, "units": None, "src": "fp_gemv_tc.cu", "sha": "4ce5acf290c2928d"},
     ("l70b", "lm_head"): {"bytes": 533911808, "units": None, "src": "fp_gemv_btc.cu", "sha": "ac6ffae462038acd"},
     ("l70b", "attn"): {"bytes": 149513984, "units": 32 * 2148, "src": "fp_attention.cu", "sha": "011e2b422a5fa35c"},
     ("l7b", "attn"): {"bytes": 81405952, "units": 8 * 612, "src": "fp_attention.cu", "sha": "011e2b422a5fa35c"},

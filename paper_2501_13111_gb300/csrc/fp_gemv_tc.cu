@@ -55,7 +55,9 @@
 
 namespace fpk {
 
-constexpr int kQ4CodeStages = 4;  // per-thread cp.async ring depth, one (own) item per stage
+// per-thread cp.async ring depth, one (own) item per stage; with 16 KB items
+// 3 stages measured 1-4 % faster than 4 (70B shapes at 32 tokens) and 5 slower
+constexpr int kQ4CodeStages = 3;
 constexpr int kQ4DeqWarps = 16;
 constexpr int kQ4MmaWarps = 2;  // MMA issuers, each with its own accumulators
 constexpr int kQ4Threads = (kQ4DeqWarps + 1 + kQ4MmaWarps) * 32;
