@@ -58,6 +58,24 @@ def test_kernel_bytes_closed_forms():
     assert kb["attn"] == pytest.approx(B * S * a["n_kv_heads"] * a["head_dim"] * 2 * 2, rel=0.02)
 
 
+def test_class_roofline_arithmetic():
+    """achieved = algorithmic bytes per launch / mean launch time, frac =
+    achieved / peak: a class with 2 launches of 100 MB in 0.1 ms in total
+    streams 2000 GB/s."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    kb = {"lin_gu": 100e6, "attn": 50e6}
+    r = bench.class_roofline("lin_gu", kb, {"lin_gu": 0.1, "attn": 0.0}, {"lin_gu": 2, "attn": 0}, 4000.0)
+    assert r["launch_ms"] == pytest.approx(0.05)
+    assert r["achieved"] == pytest.approx(2000.0)
+    assert r["frac"] == pytest.approx(0.5)
+    assert r["bytes_per_launch"] == 100e6
+    # a class that did not run reports zero rather than dividing by zero
+    z = bench.class_roofline("attn", kb, {"lin_gu": 0.1, "attn": 0.0}, {"lin_gu": 2, "attn": 0}, 4000.0)
+    assert z["achieved"] == 0.0 and z["frac"] == 0.0
+
+
 def test_source_code_sha_ignores_comments_only(tmp_path):
     """The recorded ncu traffic stays valid across comment edits of a kernel's
     source and goes stale on any code edit."""
