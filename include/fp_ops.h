@@ -67,11 +67,15 @@ enum {
  * Kernel choice depends on M, N and K: M <= 64 runs the decode GEMV (the
  * work is cut into equal ranges of (128-row block, K step), one per resident
  * CTA, and shared blocks are reduced from fp32 partials in a fixed order) --
- * on mma.sync with the codes dequantised in registers, except int4 with
- * 17 <= M <= 64 and 16-byte aligned x and codes, which runs on tcgen05 with
- * each weight expanded to bf16((q - z) s) as the prefill GEMM does; a K that
- * is not a multiple of the GEMV's K step falls back to one warp per output
- * row on the CUDA cores -- larger M the tcgen05 GEMM.  For M > 64 with int8
+ * on mma.sync with the codes dequantised in registers, except, with 16-byte
+ * aligned x and codes: int4 with 17 <= M <= 64 (K a multiple of 128), and
+ * int8 with 33 <= M <= 64 or K >= 16384, which run on tcgen05 with each
+ * weight expanded in TMEM (int4 to bf16((q - z) s) as the prefill GEMM does,
+ * int8 to the integer code, its row scale applied to the fp32 sums); bf16
+ * with 17 <= M <= 64 on matrices that give every SM at least 48 items of 32
+ * KB, which runs on tcgen05 fed by TMA; a K that is not a multiple of the
+ * GEMV's K step falls back to one warp per output row on the CUDA cores --
+ * larger M the tcgen05 GEMM.  For M > 64 with int8
  * or int4 weights the GEMM either reads a bf16 expansion of W that it writes
  * into the workspace band by band (at most 128 MB; the faster path), or, when
  * the workspace is NULL or smaller than that, dequantises the codes inside
